@@ -1,0 +1,293 @@
+/*
+ * ARCHead packed LM-head forward: plain fp64 CPU oracle.
+ *
+ * TEST INFRASTRUCTURE.  Only the test suite, the package smoke check and the
+ * benchmark's CPU-baseline leg may load or call this library.  It shares no
+ * code, header, table or helper with the CUDA path: it has its own nibble
+ * unpacking, its own fp16/bf16 decoders and its own loops.
+ *
+ * What it computes (paper, Section 3.2, Eqs. 3, 6 and 7):
+ *
+ *   W_hat[n,k] = code[n,k] * s_R[n, k/g]                       (INT4 residual)
+ *              + sum_j (qU[n,j] sU[j]) * (qV[k,j] sV[j])          (core A_c B_c)
+ *              + sum_j (qA[n,j] sA[n]) * (qB[k,j] sB[k/g, j])     (correction A_w B_w)
+ *   y[m,n]     = sum_k x[m,k] * W_hat[n,k]
+ *   ce[m]      = log sum_n exp(y[m,n]) - y[m, t_m]                (Section 4, CE)
+ *
+ * Everything is evaluated in double precision exactly as written: a dense
+ * fp64 row of W_hat is formed, then dotted with every token.  There is no
+ * blocking or reordering beyond processing one vocabulary row at a time.
+ *
+ * Readings where the paper is silent (stated once here, used throughout):
+ *  - INT4 codes are two's complement, packed along d, low nibble = even k.
+ *  - All quantisers are symmetric (no zero points); scales are IEEE fp16.
+ *  - A_w is quantised per row (one scale per vocabulary row) and B_w per
+ *    (d-group of size g, rank column); the core factors per column.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+typedef struct {
+  int64_t V, d;
+  int32_t core_rank, corr_rank, group_size, pad_;
+  const uint8_t *res_codes;      /* V x d/2                       */
+  const uint16_t *res_scales;    /* V x d/g   fp16 bits           */
+  const int8_t *core_u;          /* V x r_c                       */
+  const uint16_t *core_u_scale;  /* r_c       fp16 bits           */
+  const int8_t *core_v;          /* d x r_c                       */
+  const uint16_t *core_v_scale;  /* r_c       fp16 bits           */
+  const int8_t *corr_a;          /* V x r_r                       */
+  const uint16_t *corr_a_scale;  /* V         fp16 bits           */
+  const int8_t *corr_b;          /* d x r_r                       */
+  const uint16_t *corr_b_scale;  /* d/g x r_r fp16 bits           */
+} oracle_head;
+
+/* IEEE-754 binary16: 1 sign bit, 5 exponent bits (bias 15), 10 fraction bits. */
+double oracle_fp16_value(uint16_t h) {
+  int sign = (h >> 15) & 1;
+  int e = (h >> 10) & 0x1F;
+  int f = h & 0x3FF;
+  double v;
+  if (e == 0) {
+    v = ldexp((double)f, -24);                 /* subnormal: f * 2^-14 * 2^-10 */
+  } else if (e == 31) {
+    v = f ? NAN : INFINITY;
+  } else {
+    v = ldexp((double)(1024 + f), e - 25);     /* (1 + f/1024) * 2^(e-15) */
+  }
+  return sign ? -v : v;
+}
+
+/* bfloat16: 1 sign bit, 8 exponent bits (bias 127), 7 fraction bits. */
+double oracle_bf16_value(uint16_t b) {
+  int sign = (b >> 15) & 1;
+  int e = (b >> 7) & 0xFF;
+  int f = b & 0x7F;
+  double v;
+  if (e == 0) {
+    v = ldexp((double)f, -133);                /* f * 2^-126 * 2^-7 */
+  } else if (e == 255) {
+    v = f ? NAN : INFINITY;
+  } else {
+    v = ldexp((double)(128 + f), e - 134);     /* (1 + f/128) * 2^(e-127) */
+  }
+  return sign ? -v : v;
+}
+
+/* Signed INT4 code k of a packed row: byte k/2, low nibble for even k. */
+int oracle_int4_code(const uint8_t *row, int64_t k) {
+  int byte = row[k / 2];
+  int nib = (k % 2 == 0) ? (byte & 0x0F) : ((byte >> 4) & 0x0F);
+  return nib >= 8 ? nib - 16 : nib;
+}
+
+void oracle_fp16_values(const uint16_t *in, int64_t n, double *out) {
+  for (int64_t i = 0; i < n; ++i) out[i] = oracle_fp16_value(in[i]);
+}
+
+void oracle_bf16_values(const uint16_t *in, int64_t n, double *out) {
+  for (int64_t i = 0; i < n; ++i) out[i] = oracle_bf16_value(in[i]);
+}
+
+void oracle_unpack_int4(const uint8_t *in, int64_t ncodes, int8_t *out) {
+  for (int64_t k = 0; k < ncodes; ++k) out[k] = (int8_t)oracle_int4_code(in, k);
+}
+
+static int check_head(const oracle_head *h) {
+  if (!h || h->V < 1 || h->d < 2 || h->group_size < 1) return -1;
+  if (h->d % 2 != 0 || h->d % h->group_size != 0) return -1;
+  if (h->core_rank < 0 || h->corr_rank < 0) return -1;
+  return 0;
+}
+
+/* Dense fp64 row n of W_hat (Eq. 6 with W_d from Eq. 3), written to w[0..d). */
+static void dequant_row(const oracle_head *h, int64_t n, double *w) {
+  const int64_t d = h->d;
+  const int g = h->group_size, rc = h->core_rank, rr = h->corr_rank;
+  const int64_t G = d / g;
+  const uint8_t *codes = h->res_codes + n * (d / 2);
+  for (int64_t k = 0; k < d; ++k) {
+    double s_r = oracle_fp16_value(h->res_scales[n * G + k / g]);
+    double v = (double)oracle_int4_code(codes, k) * s_r;
+    double core = 0.0;
+    for (int j = 0; j < rc; ++j) {
+      double u = (double)h->core_u[n * rc + j] * oracle_fp16_value(h->core_u_scale[j]);
+      double b = (double)h->core_v[k * rc + j] * oracle_fp16_value(h->core_v_scale[j]);
+      core += u * b;
+    }
+    double corr = 0.0;
+    double s_a = rr > 0 ? oracle_fp16_value(h->corr_a_scale[n]) : 0.0;
+    for (int j = 0; j < rr; ++j) {
+      double a = (double)h->corr_a[n * rr + j] * s_a;
+      double b = (double)h->corr_b[k * rr + j] * oracle_fp16_value(h->corr_b_scale[(k / g) * rr + j]);
+      corr += a * b;
+    }
+    w[k] = v + core + corr;
+  }
+}
+
+int oracle_dequant_rows(const oracle_head *h, int64_t row0, int64_t nrows, double *out) {
+  if (check_head(h) || row0 < 0 || nrows < 0 || row0 + nrows > h->V) return -1;
+#pragma omp parallel for schedule(static)
+  for (int64_t i = 0; i < nrows; ++i) dequant_row(h, row0 + i, out + i * h->d);
+  return 0;
+}
+
+/*
+ * One stored component, dequantised element by element as code * scale:
+ *   0: residual      [nrows x d]    code[n,k] * s_R[n,k/g]
+ *   1: core left     [nrows x r_c]  qU[n,j] * sU[j]
+ *   2: core right    [nrows x r_c]  qV[k,j] * sV[j]         (rows are k)
+ *   3: corr left     [nrows x r_r]  qA[n,j] * sA[n]
+ *   4: corr right    [nrows x r_r]  qB[k,j] * sB[k/g,j]     (rows are k)
+ */
+int oracle_component(const oracle_head *h, int comp, int64_t row0, int64_t nrows, double *out) {
+  if (check_head(h) || row0 < 0 || nrows < 0) return -1;
+  const int64_t d = h->d;
+  const int g = h->group_size, rc = h->core_rank, rr = h->corr_rank;
+  const int64_t G = d / g;
+  int64_t limit = (comp == 2 || comp == 4) ? d : h->V;
+  if (comp < 0 || comp > 4 || row0 + nrows > limit) return -1;
+  for (int64_t i = 0; i < nrows; ++i) {
+    int64_t r = row0 + i;
+    if (comp == 0) {
+      for (int64_t k = 0; k < d; ++k)
+        out[i * d + k] = (double)oracle_int4_code(h->res_codes + r * (d / 2), k) *
+                         oracle_fp16_value(h->res_scales[r * G + k / g]);
+    } else if (comp == 1) {
+      for (int j = 0; j < rc; ++j)
+        out[i * rc + j] = (double)h->core_u[r * rc + j] * oracle_fp16_value(h->core_u_scale[j]);
+    } else if (comp == 2) {
+      for (int j = 0; j < rc; ++j)
+        out[i * rc + j] = (double)h->core_v[r * rc + j] * oracle_fp16_value(h->core_v_scale[j]);
+    } else if (comp == 3) {
+      for (int j = 0; j < rr; ++j)
+        out[i * rr + j] = (double)h->corr_a[r * rr + j] * oracle_fp16_value(h->corr_a_scale[r]);
+    } else {
+      for (int j = 0; j < rr; ++j)
+        out[i * rr + j] = (double)h->corr_b[r * rr + j] *
+                          oracle_fp16_value(h->corr_b_scale[(r / g) * rr + j]);
+    }
+  }
+  return 0;
+}
+
+/*
+ * Logits of vocabulary rows [row0, row0+nrows) for M tokens (Eq. 7):
+ *   y[m * nrows + (n - row0)] = sum_k x[m,k] * W_hat[n,k].
+ * x holds bf16 bit patterns, row-major [M x d].
+ */
+int oracle_logits(const oracle_head *h, const uint16_t *x_bits, int64_t M, int64_t row0,
+                  int64_t nrows, double *y) {
+  if (check_head(h) || M < 0 || row0 < 0 || nrows < 0 || row0 + nrows > h->V) return -1;
+  const int64_t d = h->d;
+  double *x = (double *)malloc(sizeof(double) * (size_t)(M * d + 1));
+  if (!x) return -2;
+  oracle_bf16_values(x_bits, M * d, x);
+  int failed = 0;
+#pragma omp parallel
+  {
+    double *w = (double *)malloc(sizeof(double) * (size_t)d);
+    if (!w) {
+#pragma omp atomic write
+      failed = 1;
+    }
+#pragma omp for schedule(static)
+    for (int64_t i = 0; i < nrows; ++i) {
+      if (!w) continue;
+      dequant_row(h, row0 + i, w);
+      for (int64_t m = 0; m < M; ++m) {
+        double acc = 0.0;
+        for (int64_t k = 0; k < d; ++k) acc += x[m * d + k] * w[k];
+        y[m * nrows + i] = acc;
+      }
+    }
+    free(w);
+  }
+  free(x);
+  return failed ? -2 : 0;
+}
+
+/*
+ * Per-token cross entropy over the full vocabulary (natural log):
+ *   ce[m] = max_n y + log sum_n exp(y[m,n] - max_n y) - y[m, t_m].
+ * Also returns the argmax (lowest index among equal maxima), the gap between
+ * the largest and second-largest logit, and the target logit.  A target
+ * outside [0, V) yields ce = NaN and the call returns 1.
+ */
+int oracle_ce(const oracle_head *h, const uint16_t *x_bits, int64_t M, const int32_t *targets,
+              double *ce, int64_t *argmax, double *top2_gap, double *target_logit) {
+  if (check_head(h) || M < 0) return -1;
+  const int64_t V = h->V;
+  double *y = (double *)malloc(sizeof(double) * (size_t)(M * V + 1));
+  if (!y) return -2;
+  int rc = oracle_logits(h, x_bits, M, 0, V, y);
+  if (rc) {
+    free(y);
+    return rc;
+  }
+  int bad_target = 0;
+  for (int64_t m = 0; m < M; ++m) {
+    const double *row = y + m * V;
+    double mx = row[0];
+    int64_t arg = 0;
+    for (int64_t n = 1; n < V; ++n)
+      if (row[n] > mx) { mx = row[n]; arg = n; }
+    double second = -INFINITY;
+    for (int64_t n = 0; n < V; ++n)
+      if (n != arg && row[n] > second) second = row[n];
+    double s = 0.0;
+    for (int64_t n = 0; n < V; ++n) s += exp(row[n] - mx);
+    double lse = mx + log(s);
+    int32_t t = targets[m];
+    if (t < 0 || t >= V) {
+      bad_target = 1;
+      ce[m] = NAN;
+      if (target_logit) target_logit[m] = NAN;
+    } else {
+      ce[m] = lse - row[t];
+      if (target_logit) target_logit[m] = row[t];
+    }
+    if (argmax) argmax[m] = arg;
+    if (top2_gap) top2_gap[m] = V > 1 ? mx - second : INFINITY;
+  }
+  free(y);
+  return bad_target;
+}
+
+/*
+ * Persistent storage of the packed head (Section 3.3, Eq. 10): the sum of
+ * numel * element_size over the stored components.  Two INT4 codes share one
+ * byte; every scale is a 2-byte fp16; every factor code one byte.
+ */
+int64_t oracle_packed_bytes(int64_t V, int64_t d, int64_t rc, int64_t rr, int64_t g) {
+  int64_t G = d / g;
+  int64_t bytes = 0;
+  bytes += V * d / 2;      /* residual codes        */
+  bytes += V * G * 2;      /* residual group scales */
+  bytes += V * rc;         /* core left codes       */
+  bytes += rc * 2;         /* core left scales      */
+  bytes += d * rc;         /* core right codes      */
+  bytes += rc * 2;         /* core right scales     */
+  bytes += V * rr;         /* correction left codes */
+  if (rr > 0) bytes += V * 2; /* correction row scales (absent when r_r = 0) */
+  bytes += d * rr;         /* correction right codes*/
+  bytes += G * rr * 2;     /* correction group scales */
+  return bytes;
+}
+
+/* The dense BF16 head the packed module replaces: V * d * 2 bytes. */
+int64_t oracle_dense_bf16_bytes(int64_t V, int64_t d) { return V * d * 2; }
+
+int oracle_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}

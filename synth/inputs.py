@@ -1,0 +1,158 @@
+"""Seeded generator of packed ARCHead heads, hidden states and targets.
+
+The packed head follows the component list of the paper's packed state
+dictionary (Appendix C, Table "Logical contents of the packed ARCHead state
+dictionary") in the symmetric INT8/INT4 variant used by this library:
+
+    res_codes     uint8  [V, d/2]    signed INT4 residual, two codes per byte:
+                                     byte j of row n holds k=2j in the low
+                                     nibble and k=2j+1 in the high nibble,
+                                     two's complement (-8..7)
+    res_scales    uint16 [V, d/g]    fp16 bit patterns, one per (row, group)
+    core_u        int8   [V, r_c]    core left factor codes (A_c, Eq. 3)
+    core_u_scale  uint16 [r_c]       fp16, one per column
+    core_v        int8   [d, r_c]    core right factor codes (B_c transposed)
+    core_v_scale  uint16 [r_c]       fp16, one per column
+    corr_a        int8   [V, r_r]    correction left codes (A_w, Eq. 5)
+    corr_a_scale  uint16 [V]         fp16, one per row (row-wise INT8)
+    corr_b        int8   [d, r_r]    correction right codes (B_w transposed)
+    corr_b_scale  uint16 [d/g, r_r]  fp16, one per (d-group, column)
+                                     (group-wise INT8 along d)
+
+Hidden states follow the anisotropic recipe x = z diag(s) Q with s
+log-spaced over [1e-2, 1e1], Q a Haar-random orthogonal matrix and a few
+outlier channels scaled by 20, cast to bf16 (round to nearest even).  The
+paper measures on real hidden states of its five heads (Section 4); those
+are not available here, so these seeded inputs stand in for them.
+
+Nothing in this module evaluates the head: it only draws codes, scales,
+hidden states and targets.
+"""
+
+from __future__ import annotations
+
+import dataclasses
+from typing import Dict
+
+import numpy as np
+
+
+@dataclasses.dataclass(frozen=True)
+class HeadShape:
+    """Shape metadata of one packed head (vocab V, hidden d, ranks, group)."""
+
+    V: int
+    d: int
+    core_rank: int
+    corr_rank: int
+    group_size: int
+    n_outliers: int = 4
+
+    @property
+    def groups(self) -> int:
+        return self.d // self.group_size
+
+
+# Head shapes of the paper's models (Section 4, "Models") in this library's
+# packed variant, plus a tiny head that the CPU oracle finishes in seconds.
+SHAPES: Dict[str, HeadShape] = {
+    "tiny": HeadShape(V=4096, d=512, core_rank=64, corr_rank=16, group_size=64, n_outliers=4),
+    "qwen3-8b": HeadShape(V=151936, d=4096, core_rank=128, corr_rank=32, group_size=128, n_outliers=4),
+    "gemma-4-e4b": HeadShape(V=262144, d=2560, core_rank=128, corr_rank=32, group_size=128, n_outliers=8),
+}
+
+# Element rms targets of the three parts of the head.  The paper prints no
+# weight statistics; these give logits with rms near 2 on the Qwen shape.
+_RMS_CORE = 0.008
+_RMS_RESIDUAL = 0.004
+_RMS_CORRECTION = 0.0012
+# rms of a code drawn uniformly from [-8, 7] and from [-127, 127]
+_RMS_INT4 = float(np.sqrt(np.mean(np.arange(-8, 8, dtype=np.float64) ** 2)))
+_MS_INT8 = float(np.mean(np.arange(-127, 128, dtype=np.float64) ** 2))
+
+_HEAD_STREAMS = (
+    "res_codes", "res_scales", "core_u", "core_u_scale", "core_v", "core_v_scale",
+    "corr_a", "corr_a_scale", "corr_b", "corr_b_scale",
+)
+
+
+def _streams(seed: int, names) -> Dict[str, np.random.Generator]:
+    children = np.random.SeedSequence(seed).spawn(len(names))
+    return {n: np.random.default_rng(c) for n, c in zip(names, children)}
+
+
+def _fp16_scales(rng: np.random.Generator, base: float, shape) -> np.ndarray:
+    # base * 2^U(-1/2, 1/2): a full random mantissa, rounded to fp16.
+    vals = base * np.exp2(rng.uniform(-0.5, 0.5, size=shape))
+    return vals.astype(np.float16).view(np.uint16)
+
+
+def _int8_codes(rng: np.random.Generator, shape) -> np.ndarray:
+    return rng.integers(-127, 128, size=shape, dtype=np.int8)
+
+
+def make_head(shape: HeadShape, seed: int = 0) -> Dict[str, np.ndarray]:
+    """Draw one packed head in the canonical layout described above."""
+    V, d, rc, rr, g = shape.V, shape.d, shape.core_rank, shape.corr_rank, shape.group_size
+    if d % 2 or d % g:
+        raise ValueError("d must be even and a multiple of the group size")
+    s = _streams(seed, _HEAD_STREAMS)
+    base_r = _RMS_RESIDUAL / _RMS_INT4
+    base_c = float(np.sqrt(_RMS_CORE / (np.sqrt(max(rc, 1)) * _MS_INT8)))
+    base_w = float(np.sqrt(_RMS_CORRECTION / (np.sqrt(max(rr, 1)) * _MS_INT8)))
+    head = {
+        # Uniform bytes are two independent uniform nibbles, i.e. codes
+        # uniform over [-8, 7] in two's complement.
+        "res_codes": s["res_codes"].integers(0, 256, size=(V, d // 2), dtype=np.uint8),
+        "res_scales": _fp16_scales(s["res_scales"], base_r, (V, d // g)),
+        "core_u": _int8_codes(s["core_u"], (V, rc)),
+        "core_u_scale": _fp16_scales(s["core_u_scale"], base_c, (rc,)),
+        "core_v": _int8_codes(s["core_v"], (d, rc)),
+        "core_v_scale": _fp16_scales(s["core_v_scale"], base_c, (rc,)),
+        "corr_a": _int8_codes(s["corr_a"], (V, rr)),
+        "corr_a_scale": _fp16_scales(s["corr_a_scale"], base_w, (V,)),
+        "corr_b": _int8_codes(s["corr_b"], (d, rr)),
+        "corr_b_scale": _fp16_scales(s["corr_b_scale"], base_w, (d // g, rr)),
+    }
+    return {k: np.ascontiguousarray(v) for k, v in head.items()}
+
+
+def head_nbytes_canonical(head: Dict[str, np.ndarray]) -> int:
+    """Sum of numel * element size over the canonical arrays."""
+    return int(sum(a.nbytes for a in head.values()))
+
+
+def _haar_orthogonal(rng: np.random.Generator, d: int) -> np.ndarray:
+    g = rng.standard_normal((d, d))
+    q, r = np.linalg.qr(g)
+    # Fold the signs of diag(R) into Q so that Q is Haar distributed.
+    return q * np.sign(np.diag(r))[None, :]
+
+
+def _f32_to_bf16_bits(a: np.ndarray) -> np.ndarray:
+    bits = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    rounded = (bits + 0x7FFF + ((bits >> 16) & 1)) >> 16
+    return rounded.astype(np.uint16)
+
+
+def make_hidden(d: int, M: int, seed: int = 0, n_outliers: int = 4) -> np.ndarray:
+    """Anisotropic hidden states x = z diag(s) Q, as bf16 bits [M, d].
+
+    Q and the outlier channels depend only on (seed, d); z depends on M too.
+    The outlier channels are scaled by 20 after the rotation.  The result is
+    rounded to fp32 and then to bf16, both to nearest even.
+    """
+    s = _streams(seed + 1_000_003, ("z", "q", "outlier"))
+    scales = np.logspace(-2.0, 1.0, d)
+    q = _haar_orthogonal(s["q"], d)
+    idx = s["outlier"].choice(d, size=min(n_outliers, d), replace=False)
+    z = s["z"].standard_normal((M, d))
+    x = (z * scales[None, :]) @ q
+    x[:, idx] *= 20.0
+    return _f32_to_bf16_bits(x.astype(np.float32))
+
+
+def make_targets(V: int, M: int, seed: int = 0) -> np.ndarray:
+    """Next-token targets drawn uniformly over [0, V)."""
+    rng = _streams(seed + 2_000_003, ("targets",))["targets"]
+    return rng.integers(0, V, size=M, dtype=np.int64).astype(np.int32)
