@@ -105,37 +105,93 @@ static int check_head(const oracle_head *h) {
   return 0;
 }
 
-/* Dense fp64 row n of W_hat (Eq. 6 with W_d from Eq. 3), written to w[0..d). */
-static void dequant_row(const oracle_head *h, int64_t n, double *w) {
+/*
+ * Dequantised d-side factors, decoded once per call and shared by all rows:
+ *   vdq[k*r_c + j] = qV[k,j] * sV[j]          (core right factor)
+ *   bdq[k*r_r + j] = qB[k,j] * sB[k/g, j]     (correction right factor)
+ *   su[j]          = sU[j]                     (core left column scales)
+ */
+typedef struct {
+  double *vdq, *bdq, *su;
+} side_cache;
+
+static void free_cache(side_cache *c) {
+  free(c->vdq);
+  free(c->bdq);
+  free(c->su);
+}
+
+static int make_cache(const oracle_head *h, side_cache *c) {
+  const int64_t d = h->d;
+  const int g = h->group_size, rc = h->core_rank, rr = h->corr_rank;
+  c->vdq = (double *)malloc(sizeof(double) * (size_t)(d * rc + 1));
+  c->bdq = (double *)malloc(sizeof(double) * (size_t)(d * rr + 1));
+  c->su = (double *)malloc(sizeof(double) * (size_t)(rc + 1));
+  if (!c->vdq || !c->bdq || !c->su) {
+    free_cache(c);
+    return -2;
+  }
+  for (int j = 0; j < rc; ++j) c->su[j] = oracle_fp16_value(h->core_u_scale[j]);
+  for (int64_t k = 0; k < d; ++k) {
+    for (int j = 0; j < rc; ++j)
+      c->vdq[k * rc + j] = (double)h->core_v[k * rc + j] * oracle_fp16_value(h->core_v_scale[j]);
+    for (int j = 0; j < rr; ++j)
+      c->bdq[k * rr + j] = (double)h->corr_b[k * rr + j] * oracle_fp16_value(h->corr_b_scale[(k / g) * rr + j]);
+  }
+  return 0;
+}
+
+/*
+ * Dense fp64 row n of W_hat (Eq. 6 with W_d from Eq. 3), written to w[0..d).
+ * u and a are scratch rows of r_c and r_r doubles.
+ */
+static void dequant_row(const oracle_head *h, const side_cache *c, int64_t n, double *w, double *u, double *a) {
   const int64_t d = h->d;
   const int g = h->group_size, rc = h->core_rank, rr = h->corr_rank;
   const int64_t G = d / g;
   const uint8_t *codes = h->res_codes + n * (d / 2);
+  for (int j = 0; j < rc; ++j) u[j] = (double)h->core_u[n * rc + j] * c->su[j];
+  double s_a = rr > 0 ? oracle_fp16_value(h->corr_a_scale[n]) : 0.0;
+  for (int j = 0; j < rr; ++j) a[j] = (double)h->corr_a[n * rr + j] * s_a;
   for (int64_t k = 0; k < d; ++k) {
     double s_r = oracle_fp16_value(h->res_scales[n * G + k / g]);
     double v = (double)oracle_int4_code(codes, k) * s_r;
     double core = 0.0;
-    for (int j = 0; j < rc; ++j) {
-      double u = (double)h->core_u[n * rc + j] * oracle_fp16_value(h->core_u_scale[j]);
-      double b = (double)h->core_v[k * rc + j] * oracle_fp16_value(h->core_v_scale[j]);
-      core += u * b;
-    }
+    for (int j = 0; j < rc; ++j) core += u[j] * c->vdq[k * rc + j];
     double corr = 0.0;
-    double s_a = rr > 0 ? oracle_fp16_value(h->corr_a_scale[n]) : 0.0;
-    for (int j = 0; j < rr; ++j) {
-      double a = (double)h->corr_a[n * rr + j] * s_a;
-      double b = (double)h->corr_b[k * rr + j] * oracle_fp16_value(h->corr_b_scale[(k / g) * rr + j]);
-      corr += a * b;
-    }
+    for (int j = 0; j < rr; ++j) corr += a[j] * c->bdq[k * rr + j];
     w[k] = v + core + corr;
   }
 }
 
+/* Per-thread scratch: one dense row plus the two left-factor rows. */
+static double *row_scratch(const oracle_head *h) {
+  return (double *)malloc(sizeof(double) * (size_t)(h->d + h->core_rank + h->corr_rank + 1));
+}
+
 int oracle_dequant_rows(const oracle_head *h, int64_t row0, int64_t nrows, double *out) {
   if (check_head(h) || row0 < 0 || nrows < 0 || row0 + nrows > h->V) return -1;
-#pragma omp parallel for schedule(static)
-  for (int64_t i = 0; i < nrows; ++i) dequant_row(h, row0 + i, out + i * h->d);
-  return 0;
+  side_cache c;
+  if (make_cache(h, &c)) return -2;
+  int failed = 0;
+#pragma omp parallel
+  {
+    double *scr = row_scratch(h);
+    if (!scr) {
+#pragma omp atomic write
+      failed = 1;
+    }
+#pragma omp for schedule(static)
+    for (int64_t i = 0; i < nrows; ++i) {
+      if (!scr) continue;
+      double *u = scr + h->d, *a = u + h->core_rank;
+      dequant_row(h, &c, row0 + i, scr, u, a);
+      memcpy(out + i * h->d, scr, sizeof(double) * (size_t)h->d);
+    }
+    free(scr);
+  }
+  free_cache(&c);
+  return failed ? -2 : 0;
 }
 
 /*
@@ -189,18 +245,23 @@ int oracle_logits(const oracle_head *h, const uint16_t *x_bits, int64_t M, int64
   double *x = (double *)malloc(sizeof(double) * (size_t)(M * d + 1));
   if (!x) return -2;
   oracle_bf16_values(x_bits, M * d, x);
+  side_cache c;
+  if (make_cache(h, &c)) {
+    free(x);
+    return -2;
+  }
   int failed = 0;
 #pragma omp parallel
   {
-    double *w = (double *)malloc(sizeof(double) * (size_t)d);
+    double *w = row_scratch(h);
     if (!w) {
 #pragma omp atomic write
       failed = 1;
     }
-#pragma omp for schedule(static)
+#pragma omp for schedule(dynamic, 16)
     for (int64_t i = 0; i < nrows; ++i) {
       if (!w) continue;
-      dequant_row(h, row0 + i, w);
+      dequant_row(h, &c, row0 + i, w, w + d, w + d + h->core_rank);
       for (int64_t m = 0; m < M; ++m) {
         double acc = 0.0;
         for (int64_t k = 0; k < d; ++k) acc += x[m * d + k] * w[k];
@@ -209,6 +270,7 @@ int oracle_logits(const oracle_head *h, const uint16_t *x_bits, int64_t M, int64
     }
     free(w);
   }
+  free_cache(&c);
   free(x);
   return failed ? -2 : 0;
 }

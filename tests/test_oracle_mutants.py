@@ -23,14 +23,14 @@ MUTANTS = {
     "bf16_exponent_bias": ("v = ldexp((double)(128 + f), e - 134);", "v = ldexp((double)(128 + f), e - 135);"),
     "residual_scale_group": ("double s_r = oracle_fp16_value(h->res_scales[n * G + k / g]);",
                              "double s_r = oracle_fp16_value(h->res_scales[n * G + (k / g + 1) % G]);"),
-    "core_scale_swapped": ("double u = (double)h->core_u[n * rc + j] * oracle_fp16_value(h->core_u_scale[j]);",
-                           "double u = (double)h->core_u[n * rc + j] * oracle_fp16_value(h->core_v_scale[j]);"),
-    "core_right_transposed": ("double b = (double)h->core_v[k * rc + j] * oracle_fp16_value(h->core_v_scale[j]);",
-                              "double b = (double)h->core_v[j * d + k] * oracle_fp16_value(h->core_v_scale[j]);"),
-    "corr_scale_table_transposed": ("oracle_fp16_value(h->corr_b_scale[(k / g) * rr + j]);\n      corr",
-                                    "oracle_fp16_value(h->corr_b_scale[j * G + (k / g)]);\n      corr"),
-    "corr_left_scale_per_column": ("double a = (double)h->corr_a[n * rr + j] * s_a;",
-                                   "double a = (double)h->corr_a[n * rr + j] * oracle_fp16_value(h->corr_a_scale[j]);"),
+    "core_scale_swapped": ("c->su[j] = oracle_fp16_value(h->core_u_scale[j]);",
+                           "c->su[j] = oracle_fp16_value(h->core_v_scale[j]);"),
+    "core_right_transposed": ("c->vdq[k * rc + j] = (double)h->core_v[k * rc + j]",
+                              "c->vdq[k * rc + j] = (double)h->core_v[j * d + k]"),
+    "corr_scale_table_transposed": ("h->corr_b_scale[(k / g) * rr + j]);\n  }\n  return 0;",
+                                    "h->corr_b_scale[j * (d / g) + (k / g)]);\n  }\n  return 0;"),
+    "corr_left_scale_per_column": ("a[j] = (double)h->corr_a[n * rr + j] * s_a;",
+                                   "a[j] = (double)h->corr_a[n * rr + j] * oracle_fp16_value(h->corr_a_scale[j]);"),
     "correction_dropped": ("w[k] = v + core + corr;", "w[k] = v + core;"),
     "core_sign": ("w[k] = v + core + corr;", "w[k] = v - core + corr;"),
     "hidden_reversed": ("acc += x[m * d + k] * w[k];", "acc += x[m * d + (d - 1 - k)] * w[k];"),
