@@ -1,0 +1,518 @@
+#!/usr/bin/env python3
+"""Benchmark of the packed LM-head forward (ARCHead, paper Section 3.2, Eq. 7)
+on GB300 through the library's C ABI.
+
+A step is one forward of the whole hot path -- rank-r pre-pass, INT4 residual
+stream with group promotion, low-rank epilogue, logits store -- over one batch
+of seeded synthetic hidden states already resident in device memory.  The
+default workload is the Qwen3-8B-shaped head (V=151936, d=4096, r_c=128,
+r_r=32, g=128) at M=1 token (decode); the same line also carries the decode
+sweep M=2..16, the M=4096 prefill (logits and fused cross entropy) and a dense
+BF16 cuBLAS head on the same shapes.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With --impl reference the fp64 CPU oracle is timed on the host cores on a
+bounded sample of the same workload (the baseline, not the target).
+Multi-GPU runs (torchrun, one rank per GPU) are independent replicas: the
+head does not shard in this build, so no collective is on the data path.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "LM-head tokens/s and achieved HBM GB/s (M=1) / TFLOP/s (M=4096), % of roofline"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+WORKLOADS = {
+    "qwen3-8b-decode": ("qwen3-8b", 1, "logits"),
+    "qwen3-8b-prefill": ("qwen3-8b", 4096, "logits"),
+    "qwen3-8b-prefill-ce": ("qwen3-8b", 4096, "ce"),
+    "gemma-4-e4b-decode": ("gemma-4-e4b", 1, "logits"),
+    "gemma-4-e4b-prefill": ("gemma-4-e4b", 2048, "logits"),
+    "tiny": ("tiny", 4, "logits"),
+}
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return {k: float(p[k]) for k in FALLBACK_PEAKS}, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ---------------------------------------------------------------------------
+# Algorithmic work (what the method must move or compute per call).
+# ---------------------------------------------------------------------------
+def packed_vocab_bytes(shape) -> int:
+    """Bytes of the V-indexed packed components the streaming kernel reads."""
+    V, d, rc, rr, g = shape.V, shape.d, shape.core_rank, shape.corr_rank, shape.group_size
+    return V * d // 2 + V * (d // g) * 2 + V * rc + V * rr + (V * 2 if rr else 0)
+
+
+def packed_bytes(shape) -> int:
+    """Eq. 10 over all stored components."""
+    V, d, rc, rr, g = shape.V, shape.d, shape.core_rank, shape.corr_rank, shape.group_size
+    G = d // g
+    return packed_vocab_bytes(shape) + rc * 2 + d * rc + rc * 2 + d * rr + G * rr * 2
+
+
+def call_bytes(shape, M, mode) -> int:
+    out = 2 * M * shape.V if mode == "logits" else 4 * M
+    return packed_bytes(shape) + 2 * M * shape.d + out
+
+
+def kernel_bytes(shape, M, mode) -> int:
+    """Algorithmic bytes of one launch of the streaming kernel."""
+    out = 2 * M * shape.V if mode == "logits" else 4 * M
+    return packed_vocab_bytes(shape) + 2 * M * shape.d + out
+
+
+def call_flops(shape, M) -> int:
+    r = shape.core_rank + shape.corr_rank
+    return 2 * M * shape.V * shape.d + 2 * M * (shape.V + shape.d) * r
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region.
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.idx = device_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        import tempfile
+
+        fd, self.path = tempfile.mkstemp(prefix="clocks", suffix=".csv")
+        os.close(fd)
+        try:
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=self.out, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        if hasattr(self, "out"):
+            self.out.close()
+
+    def summary(self):
+        if self.proc is None or not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 8:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+
+        def num(v):
+            try:
+                return float(v)
+            except ValueError:
+                return None
+
+        sm = [num(r[0]) for r in rows if num(r[0]) is not None]
+        mx = [num(r[1]) for r in rows if num(r[1]) is not None]
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            for name, v in zip(names, r[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        loaded = sorted(sm)[len(sm) // 4:] if len(sm) >= 4 else sm
+        return {"sm_mhz": statistics.median(loaded) if loaded else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(rows),
+                "power_w_max": max((num(r[2]) or 0.0) for r in rows)}
+
+
+# ---------------------------------------------------------------------------
+# Distributed helpers (replicas; host-side logic covered by the gloo tests).
+# ---------------------------------------------------------------------------
+def dist_env():
+    return int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), int(
+        os.environ.get("LOCAL_RANK", "0"))
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+# ---------------------------------------------------------------------------
+# Our arm.
+# ---------------------------------------------------------------------------
+class Workload:
+    def __init__(self, shape_name: str, seed: int = 0):
+        from synth import SHAPES, make_head
+
+        self.shape = SHAPES[shape_name]
+        self.head = make_head(self.shape, seed=seed)
+        self.pack = None
+
+    def open(self):
+        from paper_2608_02703_gb300 import archead
+
+        self.pack = archead.archead_pack_create(self.head, self.shape)
+        return self.pack
+
+
+def timed_loop(fn, steps: int, warmup: int, world: int):
+    import torch
+
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    return e0.elapsed_time(e1) / 1e3
+
+
+def profiled_kernels(pack, fn, steps: int):
+    """Per-kernel mean launch duration (ms) from the library's CUDA events."""
+    import torch
+
+    from paper_2608_02703_gb300 import archead
+
+    archead.archead_profile_read(pack)  # drain
+    base = {s["name"]: (s["launches"], s["total_ms"]) for s in archead.archead_profile_read(pack)}
+    archead.archead_profile_enable(pack, True)
+    for _ in range(steps):
+        fn()
+    torch.cuda.synchronize()
+    archead.archead_profile_enable(pack, False)
+    out = {}
+    for s in archead.archead_profile_read(pack):
+        l0, t0 = base.get(s["name"], (0, 0.0))
+        n, t = s["launches"] - l0, s["total_ms"] - t0
+        if n > 0:
+            out[s["name"]] = {"launches_per_step": n / steps, "mean_ms": t / n}
+    return out
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+
+    from paper_2608_02703_gb300 import archead
+    from paper_2608_02703_gb300.build import build
+    from synth import make_hidden, make_targets
+
+    build()
+    torch.cuda.set_device(local_rank)
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    peaks, peak_src = load_peaks()
+    shape_name, M, mode = WORKLOADS[args.workload]
+    if args.M:
+        M = args.M
+    wl = Workload(shape_name)
+    shape = wl.shape
+    pack = wl.open()
+    x_np = make_hidden(shape.d, M, seed=1, n_outliers=shape.n_outliers)
+    x = torch.from_numpy(x_np.view(np.int16)).cuda()
+    t_np = make_targets(shape.V, M, seed=1)
+    tgt = torch.from_numpy(t_np).cuda()
+    y = torch.empty((M, shape.V), dtype=torch.bfloat16, device="cuda")
+    ce = torch.empty(M, dtype=torch.float32, device="cuda")
+
+    def step():
+        if mode == "logits":
+            archead.archead_forward(pack, x, M, y, archead.OUT_BF16)
+        else:
+            archead.archead_forward_ce(pack, x, M, tgt, ce)
+
+    steps, warmup = args.steps, args.warmup
+    if steps is None:
+        steps = 20000 if M <= 16 else 20
+    with ClockSampler(local_rank) as clk:
+        secs = timed_loop(step, steps, warmup, world)
+    st = archead.archead_sync_status(pack)
+    if st != archead.OK:
+        raise RuntimeError(f"device error after timed loop: {archead.archead_status_string(st)}")
+    secs_max = max_over_ranks(secs, world, torch.device("cuda", local_rank))
+    tokens_s = world * M * steps / secs_max
+
+    prof = profiled_kernels(pack, step, max(3, min(steps, 2000)))
+    main_kernel = "decode" if "decode" in prof else max(prof, key=lambda k: prof[k]["mean_ms"])
+    launches_per_step = sum(v["launches_per_step"] for v in prof.values())
+    kb = kernel_bytes(shape, M, mode)
+    kms = prof[main_kernel]["mean_ms"]
+    if M <= 64:
+        achieved = kb / (kms / 1e3) / 1e9
+        roof = {"kernel": main_kernel, "bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"],
+                "unit": "GB/s", "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": None,
+                "peak_source": peak_src, "algorithmic_bytes_per_launch": kb, "mean_launch_ms": kms}
+    else:
+        fl = call_flops(shape, M) / prof[main_kernel]["launches_per_step"]
+        achieved = fl / (kms / 1e3) / 1e12
+        peak = peaks["bf16_tflops"]
+        roof = {"kernel": main_kernel, "bound": "tensor", "achieved": round(achieved, 1), "peak": peak,
+                "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "traffic": None, "peak_source": peak_src,
+                "algorithmic_flops_per_launch": fl, "mean_launch_ms": kms}
+
+    # End to end through the public host-buffer entry point.
+    e2e = None
+    if mode == "logits":
+        xh = torch.from_numpy(x_np.view(np.int16).copy()).pin_memory()
+        yh = torch.empty((M, shape.V), dtype=torch.bfloat16).pin_memory()
+        k2 = max(3, min(steps, 2000 if M <= 16 else 5))
+        for _ in range(3):
+            archead.archead_forward_host(pack, xh, M, yh, archead.OUT_BF16)
+        barrier(world)
+        t0 = time.perf_counter()
+        for _ in range(k2):
+            archead.archead_forward_host(pack, xh, M, yh, archead.OUT_BF16)
+        t_e2e = max_over_ranks(time.perf_counter() - t0, world, torch.device("cuda", local_rank))
+        e2e = {"value": round(world * M * k2 / t_e2e, 2), "unit": "tokens/s", "h2d_bytes_per_step": M * shape.d * 2,
+               "d2h_bytes_per_step": M * shape.V * 2, "steps": k2}
+
+    result = {
+        "metric": METRIC, "value": round(tokens_s, 2), "unit": "tokens/s", "n_gpus": world, "steps": steps,
+        "warmup": warmup, "ms_per_step": round(secs_max / steps * 1e3, 5), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"{shape_name} head, {'decode' if M <= 16 else 'prefill'} M={M}, "
+                               f"{'logits bf16' if mode == 'logits' else 'fused CE'}",
+                   "V": shape.V, "d": shape.d, "core_rank": shape.core_rank, "corr_rank": shape.corr_rank,
+                   "group_size": shape.group_size, "M": M, "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2: the packed head (%.1f MB) exceeds the 129 MB L2, so every "
+                         "forward streams it from HBM" % (packed_bytes(shape) / 1e6)},
+        "roofline": roof,
+        "gpu_launches": int(round(launches_per_step * steps)),
+        "kernels": {k: {"launches_per_step": v["launches_per_step"], "mean_us": round(v["mean_ms"] * 1e3, 3)}
+                    for k, v in prof.items()},
+        "e2e": e2e,
+        "clocks": clk.summary(),
+        "algorithmic": {"bytes_per_call": call_bytes(shape, M, mode), "flops_per_call": call_flops(shape, M),
+                        "gbs_per_call": round(call_bytes(shape, M, mode) / (secs_max / steps) / 1e9, 1)},
+    }
+
+    if not args.no_extras and args.workload == "qwen3-8b-decode":
+        result["decode_sweep"] = decode_sweep(pack, shape, peaks, world, local_rank)
+        result["prefill"] = prefill_block(pack, shape, peaks, world, local_rank)
+        result["dense_bf16_cublas"] = dense_comparator(shape, world, local_rank)
+    pack.close()
+    if rank == 0 and not args.no_cpu_baseline and world == 1:
+        result["cpu_baseline"] = cpu_baseline(wl, x_np, M, budget_s=args.cpu_budget)
+    return result
+
+
+def decode_sweep(pack, shape, peaks, world, local_rank):
+    import torch
+
+    from paper_2608_02703_gb300 import archead
+    from synth import make_hidden
+
+    out = []
+    for M in (1, 2, 4, 8, 16):
+        x = torch.from_numpy(make_hidden(shape.d, M, seed=2, n_outliers=shape.n_outliers).view(np.int16)).cuda()
+        y = torch.empty((M, shape.V), dtype=torch.bfloat16, device="cuda")
+        fn = lambda: archead.archead_forward(pack, x, M, y, archead.OUT_BF16)  # noqa: E731
+        k = 2000
+        secs = max_over_ranks(timed_loop(fn, k, 20, world), world, torch.device("cuda", local_rank))
+        prof = profiled_kernels(pack, fn, 500)
+        kms = prof["decode"]["mean_ms"]
+        gbs = kernel_bytes(shape, M, "logits") / (kms / 1e3) / 1e9
+        out.append({"M": M, "tokens_s": round(world * M * k / secs, 1), "us_per_call": round(secs / k * 1e6, 2),
+                    "decode_kernel_us": round(kms * 1e3, 2), "decode_gbs": round(gbs, 1),
+                    "frac_hbm": round(gbs / peaks["hbm_gbs"], 4)})
+    return out
+
+
+def prefill_block(pack, shape, peaks, world, local_rank):
+    import torch
+
+    from paper_2608_02703_gb300 import archead
+    from synth import make_hidden, make_targets
+
+    M = 4096
+    x = torch.from_numpy(make_hidden(shape.d, M, seed=3, n_outliers=shape.n_outliers).view(np.int16)).cuda()
+    y = torch.empty((M, shape.V), dtype=torch.bfloat16, device="cuda")
+    tgt = torch.from_numpy(make_targets(shape.V, M, seed=3)).cuda()
+    ce = torch.empty(M, dtype=torch.float32, device="cuda")
+    res = {"M": M}
+    for mode, fn in (("logits", lambda: archead.archead_forward(pack, x, M, y, archead.OUT_BF16)),
+                     ("ce", lambda: archead.archead_forward_ce(pack, x, M, tgt, ce))):
+        k = 5
+        secs = max_over_ranks(timed_loop(fn, k, 3, world), world, torch.device("cuda", local_rank))
+        tf = call_flops(shape, M) / (secs / k) / 1e12
+        res[mode] = {"tokens_s": round(world * M * k / secs, 1), "ms_per_call": round(secs / k * 1e3, 3),
+                     "tflops": round(tf, 1), "frac_bf16_peak": round(tf / peaks["bf16_tflops"], 4)}
+    st = archead.archead_sync_status(pack)
+    res["status"] = archead.archead_status_string(st)
+    return res
+
+
+def dense_comparator(shape, world, local_rank):
+    """Dense BF16 V x d head through cuBLAS (torch.matmul) on the same shapes."""
+    import torch
+
+    g = torch.Generator(device="cuda")
+    g.manual_seed(0)
+    W = (torch.randn((shape.V, shape.d), generator=g, device="cuda", dtype=torch.float32) * 0.01).to(torch.bfloat16)
+    res = {}
+    for M in (1, 16, 4096):
+        x = torch.randn((M, shape.d), generator=g, device="cuda", dtype=torch.float32).to(torch.bfloat16)
+        fn = lambda: torch.matmul(x, W.t())  # noqa: E731
+        k = 200 if M <= 16 else 10
+        secs = max_over_ranks(timed_loop(fn, k, 5, world), world, torch.device("cuda", local_rank))
+        res[f"M={M}"] = {"tokens_s": round(world * M * k / secs, 1), "us_per_call": round(secs / k * 1e6, 2),
+                         "tflops": round(2 * M * shape.V * shape.d / (secs / k) / 1e12, 2)}
+    del W
+    torch.cuda.empty_cache()
+    return res
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (baseline leg and reference arm).
+# ---------------------------------------------------------------------------
+def oracle_rows_time(head, shape, x_np, rows: int) -> float:
+    import oracle
+
+    t0 = time.perf_counter()
+    oracle.logits(head, shape, x_np, row0=0, nrows=rows)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(wl, x_np, M, budget_s: float = 15.0):
+    """Time the oracle as it stands on a bounded sample of vocabulary rows."""
+    import oracle
+
+    shape = wl.shape
+    rows = min(shape.V, 1024)
+    t = oracle_rows_time(wl.head, shape, x_np, rows)
+    while t < budget_s / 4 and rows < shape.V:
+        rows = min(shape.V, int(rows * max(2.0, budget_s / 2 / max(t, 1e-3))))
+        t = oracle_rows_time(wl.head, shape, x_np, rows)
+    full = t * shape.V / rows
+    return {"value": round(M / full, 4), "unit": "tokens/s", "cores": oracle.threads(), "kind": "oracle",
+            "sample": f"fp64 oracle logits of the first {rows} of {shape.V} vocabulary rows for M={M} token(s), "
+                      f"{t:.2f} s; scaled by V/rows to a full forward"}
+
+
+def run_reference(args, rank, world):
+    import oracle
+    from synth import make_hidden
+
+    if rank != 0:
+        return None
+    oracle.build()
+    shape_name, M, mode = WORKLOADS[args.workload]
+    if args.M:
+        M = args.M
+    wl = Workload(shape_name)
+    shape = wl.shape
+    x_np = make_hidden(shape.d, M, seed=1, n_outliers=shape.n_outliers)
+    steps = args.steps if args.steps is not None else 20
+    warmup = args.warmup
+    # Size one step so that the whole run takes about two minutes.
+    t1 = oracle_rows_time(wl.head, shape, x_np, 256)
+    per_row = max(t1 / 256, 1e-7)
+    rows = int(max(16, min(shape.V, (args.ref_budget / max(steps + warmup, 1)) / per_row)))
+    for _ in range(warmup):
+        oracle_rows_time(wl.head, shape, x_np, rows)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        oracle_rows_time(wl.head, shape, x_np, rows)
+    secs = time.perf_counter() - t0
+    tokens_s = M * steps * rows / shape.V / secs
+    sample = (f"each step: fp64 oracle logits of {rows} of {shape.V} vocabulary rows for M={M} token(s) "
+              f"(a {rows / shape.V:.4f} fraction of one forward)")
+    return {
+        "metric": METRIC, "value": round(tokens_s, 4), "unit": "tokens/s", "n_gpus": world, "steps": steps,
+        "warmup": warmup, "ms_per_step": round(secs / steps * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+        "config": {"workload": f"{shape_name} head, {'decode' if M <= 16 else 'prefill'} M={M}, "
+                               f"{'logits' if mode == 'logits' else 'CE'}", "V": shape.V, "d": shape.d, "M": M},
+        "cpu_baseline": {"value": round(tokens_s, 4), "unit": "tokens/s", "cores": oracle.threads(),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(tokens_s, 4), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=None)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="qwen3-8b-decode")
+    ap.add_argument("--M", type=int, default=None)
+    ap.add_argument("--no-extras", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=15.0)
+    ap.add_argument("--ref-budget", type=float, default=90.0)
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    rank, world, local_rank = dist_env()
+    if args.impl == "reference":
+        res = run_reference(args, rank, world)
+    else:
+        res = run_ours(args, rank, world, local_rank)
+    if rank == 0 and res is not None:
+        print(json.dumps(res), flush=True)
+    if world > 1 and args.impl == "ours":
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,225 @@
+/*
+ * archead.h -- C ABI of the GB300 (sm_103a) packed LM-head forward.
+ *
+ * The packed head replaces a dense output projection W (V x d) by
+ *
+ *   W_hat = W_d + A_w B_w,      W_d = Q(A_c) Q(B_c) + Q_SC4(W - A_c B_c)
+ *
+ * (paper, Section 3.2, Eqs. 3 and 6) and the forward evaluates
+ *
+ *   Y_hat = H W_d^T + (H B_w^T) A_w^T                       (Eq. 7)
+ *
+ * without ever forming a dense W_hat: the INT4 residual is streamed and
+ * dequantised tile by tile, and both rank-r branches are applied as factored
+ * products.  In this ABI, H is called x (M tokens x d) and the factors are
+ *
+ *   core_u = A_c (V x r_c), core_v = B_c^T (d x r_c),
+ *   corr_a = A_w (V x r_r), corr_b = B_w^T (d x r_r).
+ *
+ * Conventions for every entry point:
+ *  - Nothing throws across the ABI; every call returns an archead_status.
+ *  - Argument and shape checks are synchronous and happen before any work is
+ *    queued.  M == 0 is a valid no-op.
+ *  - "stream" is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *    Device work is queued on it; results are ready when it completes.
+ *  - Device pointers must be 16-byte aligned; x rows must be contiguous.
+ *  - A pack may be used by one stream at a time (the workspace it owns for
+ *    the pre-pass and the cross-entropy partials is not shared safely between
+ *    concurrent calls).  Different packs are independent.
+ *  - Faults detected on the device (an out-of-range target, a pipeline wait
+ *    that gave up) are latched in a per-pack device error word and reported
+ *    by archead_sync_status().
+ */
+#ifndef ARCHEAD_H_
+#define ARCHEAD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define ARCHEAD_API __attribute__((visibility("default")))
+#else
+#define ARCHEAD_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct archead_pack archead_pack; /* opaque, owned by the library */
+
+typedef enum {
+  ARCHEAD_OK = 0,
+  ARCHEAD_ERR_INVALID_ARG = 1,    /* NULL pointer, bad shape, misaligned pointer      */
+  ARCHEAD_ERR_UNSUPPORTED = 2,    /* valid request outside the supported envelope     */
+  ARCHEAD_ERR_OOM = 3,            /* a device allocation failed                       */
+  ARCHEAD_ERR_CUDA = 4,           /* a CUDA runtime call failed (see last_error)      */
+  ARCHEAD_ERR_DEVICE_TIMEOUT = 5, /* a bounded pipeline wait gave up on the device    */
+  ARCHEAD_ERR_TARGET_RANGE = 6    /* a CE target was outside [0, V); its ce is NaN     */
+} archead_status;
+
+typedef enum {
+  ARCHEAD_OUT_BF16 = 0, /* logits rounded to bf16 (nearest even) from fp32 accumulators */
+  ARCHEAD_OUT_FP32 = 1  /* logits as the fp32 accumulators                               */
+} archead_out_dtype;
+
+typedef enum {
+  ARCHEAD_PATH_AUTO = 0,    /* decode kernel for M <= 16, prefill kernel above          */
+  ARCHEAD_PATH_DECODE = 1,  /* memory-bound decode kernel (tokens taken 16 at a time)   */
+  ARCHEAD_PATH_PREFILL = 2  /* tensor-core prefill kernel                               */
+} archead_path;
+
+/*
+ * The packed head in its canonical layout (paper, Appendix C, Table
+ * "Logical contents of the packed ARCHead state dictionary"; Section 3.2).
+ * Symmetric quantisers throughout (no zero points); every scale is an IEEE
+ * fp16 bit pattern.  Pointers may be host or device memory (anything CUDA's
+ * unified addressing resolves); they are read during archead_pack_create only.
+ *
+ *   res_codes    uint8 [V][d/2]   signed INT4 residual Q_SC4(W - A_c B_c),
+ *                                 two's complement, packed along d: byte j of
+ *                                 row n holds k = 2j (low nibble) and k = 2j+1
+ *   res_scales   fp16  [V][d/g]   one scale per (row, group of g along d)
+ *   core_u       int8  [V][r_c]   core left factor codes,  core_u_scale fp16 [r_c] (per column)
+ *   core_v       int8  [d][r_c]   core right factor codes, core_v_scale fp16 [r_c] (per column)
+ *   corr_a       int8  [V][r_r]   correction left codes,   corr_a_scale fp16 [V]   (per row)
+ *   corr_b       int8  [d][r_r]   correction right codes,  corr_b_scale fp16 [d/g][r_r]
+ *                                 (per group of g along d and rank column)
+ *
+ * Dequantised values are code * scale, e.g. W_hat[n,k] =
+ *   code[n,k] s_R[n,k/g] + sum_j core_u[n,j] su[j] core_v[k,j] sv[j]
+ *                        + sum_j corr_a[n,j] sa[n] corr_b[k,j] sb[k/g,j].
+ * A rank of 0 drops that branch (its pointers may then be NULL): r_c = r_r = 0
+ * is the plain group-wise INT4 head, r_r = 0 the "core only" variant.
+ *
+ * Supported envelope: V >= 1; d a multiple of 64 and of g; g in {32, 64,
+ * 128, 256}; 0 <= r_c, r_r <= 256.
+ */
+typedef struct {
+  int64_t vocab;       /* V */
+  int64_t hidden;      /* d */
+  int32_t core_rank;   /* r_c */
+  int32_t corr_rank;   /* r_r */
+  int32_t group_size;  /* g */
+  int32_t reserved;    /* must be 0 */
+  const void *res_codes;
+  const void *res_scales;
+  const void *core_u;
+  const void *core_u_scale;
+  const void *core_v;
+  const void *core_v_scale;
+  const void *corr_a;
+  const void *corr_a_scale;
+  const void *corr_b;
+  const void *corr_b_scale;
+} archead_desc;
+
+/*
+ * Build a pack on the current CUDA device: copies every component into
+ * library-owned device memory and re-tiles it into the kernels' layouts
+ * (one pass on the device).  Returns after the pack is ready; the caller's
+ * buffers may be freed as soon as it returns.  On failure *out is NULL.
+ */
+ARCHEAD_API archead_status archead_pack_create(const archead_desc *desc, void *stream, archead_pack **out);
+
+/* Free a pack and everything it owns.  NULL is a no-op. */
+ARCHEAD_API void archead_destroy(archead_pack *pack);
+
+/*
+ * Logits (Eq. 7): logits[m][n] = sum_k x[m][k] W_hat[n][k] for m < M, n < V.
+ *   x       device, bf16 [M][d] row-major
+ *   logits  device, [M][V] row-major, bf16 or fp32 per out_dtype
+ * fp32 accumulation throughout; bf16 output is rounded once at the end.
+ */
+ARCHEAD_API archead_status archead_forward(archead_pack *pack, const void *x, int64_t M, void *logits,
+                               archead_out_dtype out_dtype, void *stream);
+
+/* archead_forward with an explicit kernel choice (for crossover sweeps and tests). */
+ARCHEAD_API archead_status archead_forward_path(archead_pack *pack, const void *x, int64_t M, void *logits,
+                                    archead_out_dtype out_dtype, archead_path path, void *stream);
+
+/*
+ * Per-token cross entropy in nats (paper, Section 4, "Data and metrics"):
+ *   ce[m] = log sum_n exp(y[m][n]) - y[m][targets[m]],   y = logits of Eq. 7,
+ * computed from the fp32 accumulators with an online max / sum of exp over
+ * vocabulary tiles; no V-wide logits are written to memory.
+ *   x        device, bf16 [M][d];  targets device, int32 [M];  ce device, fp32 [M]
+ * A target outside [0, V) gives ce = NaN and latches ARCHEAD_ERR_TARGET_RANGE.
+ */
+ARCHEAD_API archead_status archead_forward_ce(archead_pack *pack, const void *x, int64_t M, const int32_t *targets,
+                                  float *ce, void *stream);
+
+ARCHEAD_API archead_status archead_forward_ce_path(archead_pack *pack, const void *x, int64_t M, const int32_t *targets,
+                                       float *ce, archead_path path, void *stream);
+
+/*
+ * End-to-end call with HOST buffers: copies x (host, bf16 [M][d]) to the
+ * device, runs archead_forward, copies the logits back to logits_host
+ * ([M][V], bf16 or fp32) and waits for the stream.  Pinned host memory
+ * makes the copies asynchronous with respect to other host work.
+ */
+ARCHEAD_API archead_status archead_forward_host(archead_pack *pack, const void *x_host, int64_t M, void *logits_host,
+                                    archead_out_dtype out_dtype, void *stream);
+
+/*
+ * Persistent storage of the packed head (paper, Section 3.3, Eq. 10): the
+ * sum of numel * element_size over the stored components listed above.  The
+ * correction's row scales count only when r_r > 0.
+ */
+ARCHEAD_API int64_t archead_pack_bytes(const archead_pack *pack);
+
+/* Bytes of device memory the pack holds now: tiled copies, padding and workspace. */
+ARCHEAD_API int64_t archead_device_bytes(const archead_pack *pack);
+
+/*
+ * Dequantise rows [row0, row0 + nrows) of one stored component with the
+ * kernels' own device unpacking, as fp32 code * scale (exact):
+ *   0 residual [nrows][d]   1 core_u [nrows][r_c]   2 core_v [nrows][r_c] (rows are k)
+ *   3 corr_a  [nrows][r_r]  4 corr_b [nrows][r_r] (rows are k)
+ * out is device memory.
+ */
+ARCHEAD_API archead_status archead_debug_dequant(const archead_pack *pack, int component, int64_t row0, int64_t nrows,
+                                     float *out, void *stream);
+
+/*
+ * Wait for the stream, then read and clear the pack's device error word.
+ * Returns ARCHEAD_OK, ARCHEAD_ERR_TARGET_RANGE, ARCHEAD_ERR_DEVICE_TIMEOUT or
+ * ARCHEAD_ERR_CUDA.
+ */
+ARCHEAD_API archead_status archead_sync_status(archead_pack *pack, void *stream);
+
+/*
+ * Upper bound, in SM clock cycles, on every pipeline wait inside the
+ * kernels (default about one second).  A wait that exceeds it latches
+ * ARCHEAD_ERR_DEVICE_TIMEOUT and its block returns early.
+ */
+ARCHEAD_API archead_status archead_set_wait_budget(archead_pack *pack, int64_t cycles);
+
+/*
+ * Launch one block whose only job is a bounded wait on a barrier that
+ * nothing completes, so the timeout path can be tested without hanging or
+ * faulting the device.  Returns after queueing it; follow with
+ * archead_sync_status() to read ARCHEAD_ERR_DEVICE_TIMEOUT.
+ */
+ARCHEAD_API archead_status archead_debug_wait_timeout(archead_pack *pack, void *stream);
+
+/* Per-kernel timing with CUDA events on the launch stream (off by default). */
+typedef struct {
+  const char *name;  /* static string */
+  int64_t launches;
+  double total_ms;
+} archead_kernel_stat;
+
+ARCHEAD_API archead_status archead_profile_enable(archead_pack *pack, int enable);
+/* Collect timings of completed launches; returns the number of entries written. */
+ARCHEAD_API int archead_profile_read(archead_pack *pack, archead_kernel_stat *out, int max_entries);
+
+ARCHEAD_API const char *archead_status_string(archead_status status);
+/* Message of the last CUDA error seen by this thread (empty if none). */
+ARCHEAD_API const char *archead_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ARCHEAD_H_ */

@@ -1,0 +1,498 @@
+// Host side of the C ABI declared in include/archead.h: argument checks, pack
+// construction, workspace management, kernel sequencing and error reporting.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstring>
+#include <string>
+
+#include "device.cuh"
+#include "internal.h"
+
+using namespace archead;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+archead_status cuda_status(cudaError_t e) {
+  g_last_error = cudaGetErrorString(e);
+  return e == cudaErrorMemoryAllocation ? ARCHEAD_ERR_OOM : ARCHEAD_ERR_CUDA;
+}
+
+#define AH_CUDA(call)                                  \
+  do {                                                 \
+    cudaError_t e_ = (call);                           \
+    if (e_ != cudaSuccess) return cuda_status(e_);     \
+  } while (0)
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
+
+template <typename T>
+cudaError_t dev_alloc(archead_pack *p, T **ptr, size_t bytes) {
+  *ptr = nullptr;
+  if (bytes == 0) return cudaSuccess;
+  cudaError_t e = cudaMalloc(reinterpret_cast<void **>(ptr), bytes);
+  if (e == cudaSuccess) p->owned_bytes += (int64_t)bytes;
+  return e;
+}
+
+void free_pack(archead_pack *p) {
+  if (!p) return;
+  void *bufs[] = {p->codes, p->scales, p->lr_codes, p->s_a, p->q_v, p->q_b, p->s_u,
+                  p->s_v,   p->s_b,    p->err,      p->ws,  p->xh_dev, p->yh_dev};
+  for (void *b : bufs)
+    if (b) cudaFree(b);
+  for (auto &t : p->timers)
+    for (auto &pr : t.pending) {
+      cudaEventDestroy(pr.first);
+      cudaEventDestroy(pr.second);
+    }
+  delete p;
+}
+
+// Workspace carve-out: consecutive 256-byte aligned regions.
+struct Carve {
+  size_t off = 0;
+  size_t take(size_t bytes) {
+    size_t o = off;
+    off += (bytes + 255) / 256 * 256;
+    return o;
+  }
+};
+
+cudaError_t ensure_workspace(archead_pack *p, size_t bytes, cudaStream_t s) {
+  if (bytes <= p->ws_bytes) return cudaSuccess;
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return e;
+  if (p->ws) {
+    cudaFree(p->ws);
+    p->owned_bytes -= (int64_t)p->ws_bytes;
+    p->ws = nullptr;
+    p->ws_bytes = 0;
+  }
+  size_t want = std::max(bytes, (size_t)1 << 20);
+  e = cudaMalloc(&p->ws, want);
+  if (e != cudaSuccess) return e;
+  p->ws_bytes = want;
+  p->owned_bytes += (int64_t)want;
+  return cudaSuccess;
+}
+
+struct ForwardPlan {
+  PrepassParams pp{};
+  size_t ce_part_off = 0, tlogit_off = 0, total = 0;
+  int nchunks = 0;
+};
+
+// Lay out the workspace of one forward over M tokens on the decode path.
+ForwardPlan plan_decode(archead_pack *p, int64_t M, bool ce) {
+  ForwardPlan f;
+  Carve c;
+  const int nsplit = (p->d + kPrepassKSplit - 1) / kPrepassKSplit;
+  f.nchunks = (int)((M + kDecodeMaxTokens - 1) / kDecodeMaxTokens);
+  size_t partial = c.take((size_t)nsplit * M * std::max(p->lr, 1) * sizeof(float));
+  size_t ts = c.take((size_t)f.nchunks * std::max(p->nls, 1) * 1024);
+  size_t xs = c.take((size_t)f.nchunks * 32 * p->d);
+  if (ce) {
+    f.ce_part_off = c.take((size_t)decode_num_units(p) * decode_parts_per_unit() * M * sizeof(float2));
+    f.tlogit_off = c.take((size_t)M * sizeof(float));
+  }
+  f.total = c.off;
+  f.pp.partial = reinterpret_cast<float *>(partial);  // offsets; rebased once the workspace exists
+  f.pp.ts = reinterpret_cast<uint32_t *>(ts);
+  f.pp.xs = reinterpret_cast<uint32_t *>(xs);
+  return f;
+}
+
+template <typename T>
+T *rebase(void *base, T *off) {
+  return reinterpret_cast<T *>(static_cast<char *>(base) + reinterpret_cast<uintptr_t>(off));
+}
+
+archead_status check_forward_args(archead_pack *p, const void *x, int64_t M, const void *out) {
+  if (!p || M < 0) return ARCHEAD_ERR_INVALID_ARG;
+  if (M == 0) return ARCHEAD_OK;
+  if (!x || !out || !aligned16(x) || !aligned16(out)) return ARCHEAD_ERR_INVALID_ARG;
+  if (M > (int64_t)1 << 30) return ARCHEAD_ERR_UNSUPPORTED;
+  return ARCHEAD_OK;
+}
+
+// Decode path over M tokens, 16 at a time.  out == nullptr selects CE mode.
+archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
+                          const int32_t *targets, float *ce, cudaStream_t s) {
+  if (!decode_supported(p->d, p->nls)) return ARCHEAD_ERR_UNSUPPORTED;
+  const bool ce_mode = out == nullptr;
+  ForwardPlan f = plan_decode(p, M, ce_mode);
+  AH_CUDA(ensure_workspace(p, f.total, s));
+  PrepassParams pp{};
+  pp.x = static_cast<const uint16_t *>(x);
+  pp.q_v = p->q_v;
+  pp.q_b = p->q_b;
+  pp.s_b = p->s_b;
+  pp.s_u = p->s_u;
+  pp.s_v = p->s_v;
+  pp.M = (int)M;
+  pp.d = p->d;
+  pp.g = p->g;
+  pp.rc = p->rc;
+  pp.rr = p->rr;
+  pp.rcp = p->rcp;
+  pp.rrp = p->rrp;
+  pp.lr = p->lr;
+  pp.partial = rebase(p->ws, f.pp.partial);
+  pp.ts = rebase(p->ws, f.pp.ts);
+  pp.xs = rebase(p->ws, f.pp.xs);
+  pp.T = nullptr;
+  AH_CUDA(launch_prepass(pp, s, p));
+
+  DecodeParams dp{};
+  dp.codes = p->codes;
+  dp.scales = p->scales;
+  dp.lr_codes = p->lr_codes;
+  dp.s_a = p->s_a;
+  dp.V = p->V;
+  dp.num_tiles = p->num_tiles;
+  dp.d = p->d;
+  dp.G = p->G;
+  dp.g = p->g;
+  dp.g_shift = 0;
+  while ((16 << dp.g_shift) < p->g) ++dp.g_shift;
+  dp.nls = p->nls;
+  dp.nls_core = p->nls_core;
+  dp.out = out;
+  dp.out_fp32 = out_fp32;
+  dp.targets = targets;
+  dp.ce_part = ce_mode ? rebase(p->ws, reinterpret_cast<float2 *>(f.ce_part_off)) : nullptr;
+  dp.ce_tlogit = ce_mode ? rebase(p->ws, reinterpret_cast<float *>(f.tlogit_off)) : nullptr;
+  dp.M_total = (int)M;
+  dp.err = p->err;
+  dp.wait_budget = p->wait_budget;
+  const int grid = std::min(decode_num_units(p), p->sm_count);
+  for (int c = 0; c < f.nchunks; ++c) {
+    dp.m0 = c * kDecodeMaxTokens;
+    dp.M = (int)std::min<int64_t>(kDecodeMaxTokens, M - dp.m0);
+    dp.NT = dp.M > 8 ? 2 : 1;
+    dp.xs = pp.xs + (size_t)c * 8 * p->d;
+    dp.ts = pp.ts + (size_t)c * p->nls * 256;
+    cudaEvent_t ev = nullptr;
+    timer_begin(p, "decode", s, &ev);
+    cudaError_t e = launch_decode(dp, grid, s);
+    timer_end(p, "decode", s, ev);
+    if (e != cudaSuccess) return cuda_status(e);
+  }
+  if (ce_mode) {
+    cudaEvent_t ev = nullptr;
+    timer_begin(p, "ce_finalize", s, &ev);
+    cudaError_t e = launch_ce_finalize(dp.ce_part, decode_num_units(p) * decode_parts_per_unit(), dp.ce_tlogit,
+                                       targets, p->V, (int)M, ce, p->err, s);
+    timer_end(p, "ce_finalize", s, ev);
+    if (e != cudaSuccess) return cuda_status(e);
+  }
+  return ARCHEAD_OK;
+}
+
+archead_status run_forward(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
+                           const int32_t *targets, float *ce, archead_path path, cudaStream_t s) {
+  if (path != ARCHEAD_PATH_AUTO && path != ARCHEAD_PATH_DECODE && path != ARCHEAD_PATH_PREFILL)
+    return ARCHEAD_ERR_INVALID_ARG;
+  AH_CUDA(cudaSetDevice(p->device));
+  // The tensor-core prefill kernel takes M > 16 when available; the decode
+  // kernel serves every M, sixteen tokens per pass.
+  return run_decode(p, x, M, out, out_fp32, targets, ce, s);
+}
+
+}  // namespace
+
+namespace archead {
+
+void timer_begin(archead_pack *p, const char *name, cudaStream_t s, cudaEvent_t *ev0) {
+  *ev0 = nullptr;
+  if (!p || !p->profiling) return;
+  if (cudaEventCreate(ev0) != cudaSuccess) {
+    *ev0 = nullptr;
+    return;
+  }
+  cudaEventRecord(*ev0, s);
+}
+
+void timer_end(archead_pack *p, const char *name, cudaStream_t s, cudaEvent_t ev0) {
+  if (!p || !p->profiling || !ev0) return;
+  cudaEvent_t ev1;
+  if (cudaEventCreate(&ev1) != cudaSuccess) {
+    cudaEventDestroy(ev0);
+    return;
+  }
+  cudaEventRecord(ev1, s);
+  for (auto &t : p->timers)
+    if (std::strcmp(t.name, name) == 0) {
+      t.pending.emplace_back(ev0, ev1);
+      return;
+    }
+  KernelTimer kt;
+  kt.name = name;
+  kt.pending.emplace_back(ev0, ev1);
+  p->timers.push_back(kt);
+}
+
+}  // namespace archead
+
+extern "C" {
+
+archead_status archead_pack_create(const archead_desc *desc, void *stream, archead_pack **out) {
+  if (!out) return ARCHEAD_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!desc) return ARCHEAD_ERR_INVALID_ARG;
+  const int64_t V = desc->vocab, d = desc->hidden;
+  const int rc = desc->core_rank, rr = desc->corr_rank, g = desc->group_size;
+  if (V < 1 || d < 64 || d % 64 != 0 || desc->reserved != 0) return ARCHEAD_ERR_INVALID_ARG;
+  if (!(g == 32 || g == 64 || g == 128 || g == 256) || d % g != 0) return ARCHEAD_ERR_INVALID_ARG;
+  if (rc < 0 || rr < 0 || rc > 256 || rr > 256) return ARCHEAD_ERR_INVALID_ARG;
+  if (d > (1 << 20) || V > ((int64_t)1 << 31) - 256) return ARCHEAD_ERR_UNSUPPORTED;
+  if (!desc->res_codes || !desc->res_scales) return ARCHEAD_ERR_INVALID_ARG;
+  if (rc > 0 && (!desc->core_u || !desc->core_u_scale || !desc->core_v || !desc->core_v_scale))
+    return ARCHEAD_ERR_INVALID_ARG;
+  if (rr > 0 && (!desc->corr_a || !desc->corr_a_scale || !desc->corr_b || !desc->corr_b_scale))
+    return ARCHEAD_ERR_INVALID_ARG;
+
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  archead_pack *p = new (std::nothrow) archead_pack();
+  if (!p) return ARCHEAD_ERR_OOM;
+  auto fail = [&](cudaError_t e) {
+    archead_status st = cuda_status(e);
+    free_pack(p);
+    return st;
+  };
+  cudaError_t e = cudaGetDevice(&p->device);
+  if (e != cudaSuccess) return fail(e);
+  e = cudaDeviceGetAttribute(&p->sm_count, cudaDevAttrMultiProcessorCount, p->device);
+  if (e != cudaSuccess) return fail(e);
+  p->V = V;
+  p->d = (int)d;
+  p->rc = rc;
+  p->rr = rr;
+  p->g = g;
+  p->G = (int)(d / g);
+  p->num_tiles = (int)((V + kTileRows - 1) / kTileRows);
+  p->V_pad = (int64_t)p->num_tiles * kTileRows;
+  p->rcp = (int)round_up(rc, 32);
+  p->rrp = (int)round_up(rr, 32);
+  p->lr = p->rcp + p->rrp;
+  p->nls = p->lr / 16;
+  p->nls_core = p->rcp / 16;
+
+  const size_t G = p->G;
+  if ((e = dev_alloc(p, &p->codes, (size_t)p->V_pad * d / 2)) != cudaSuccess) return fail(e);
+  if ((e = dev_alloc(p, &p->scales, (size_t)p->V_pad * G * 2)) != cudaSuccess) return fail(e);
+  if ((e = dev_alloc(p, &p->lr_codes, (size_t)p->num_tiles * p->nls * kLrStepBytes)) != cudaSuccess) return fail(e);
+  if ((e = dev_alloc(p, &p->s_a, (size_t)p->V_pad * 2)) != cudaSuccess) return fail(e);
+  if ((e = dev_alloc(p, &p->q_v, (size_t)d * rc)) != cudaSuccess) return fail(e);
+  if ((e = dev_alloc(p, &p->q_b, (size_t)d * rr)) != cudaSuccess) return fail(e);
+  if ((e = dev_alloc(p, &p->s_u, (size_t)rc * 2)) != cudaSuccess) return fail(e);
+  if ((e = dev_alloc(p, &p->s_v, (size_t)rc * 2)) != cudaSuccess) return fail(e);
+  if ((e = dev_alloc(p, &p->s_b, G * rr * 2)) != cudaSuccess) return fail(e);
+  if ((e = dev_alloc(p, &p->err, 16)) != cudaSuccess) return fail(e);
+  if ((e = cudaMemsetAsync(p->err, 0, 16, s)) != cudaSuccess) return fail(e);
+
+  // Canonical components: the V-indexed ones pass through temporaries on the
+  // device and are re-tiled; the d-indexed ones are copied as they are.
+  uint8_t *t_codes = nullptr, *t_scales = nullptr, *t_u = nullptr, *t_a = nullptr, *t_sa = nullptr;
+  auto free_tmp = [&]() {
+    for (void *b : {(void *)t_codes, (void *)t_scales, (void *)t_u, (void *)t_a, (void *)t_sa})
+      if (b) cudaFree(b);
+  };
+  auto tmp_copy = [&](uint8_t **dst, const void *src, size_t bytes) -> cudaError_t {
+    if (bytes == 0) return cudaSuccess;
+    cudaError_t e2 = cudaMalloc(reinterpret_cast<void **>(dst), bytes);
+    if (e2 != cudaSuccess) return e2;
+    return cudaMemcpyAsync(*dst, src, bytes, cudaMemcpyDefault, s);
+  };
+  e = tmp_copy(&t_codes, desc->res_codes, (size_t)V * d / 2);
+  if (e == cudaSuccess) e = tmp_copy(&t_scales, desc->res_scales, (size_t)V * G * 2);
+  if (e == cudaSuccess && rc > 0) e = tmp_copy(&t_u, desc->core_u, (size_t)V * rc);
+  if (e == cudaSuccess && rr > 0) e = tmp_copy(&t_a, desc->corr_a, (size_t)V * rr);
+  if (e == cudaSuccess && rr > 0) e = tmp_copy(&t_sa, desc->corr_a_scale, (size_t)V * 2);
+  if (e == cudaSuccess && rc > 0) e = cudaMemcpyAsync(p->q_v, desc->core_v, (size_t)d * rc, cudaMemcpyDefault, s);
+  if (e == cudaSuccess && rc > 0) e = cudaMemcpyAsync(p->s_u, desc->core_u_scale, (size_t)rc * 2, cudaMemcpyDefault, s);
+  if (e == cudaSuccess && rc > 0) e = cudaMemcpyAsync(p->s_v, desc->core_v_scale, (size_t)rc * 2, cudaMemcpyDefault, s);
+  if (e == cudaSuccess && rr > 0) e = cudaMemcpyAsync(p->q_b, desc->corr_b, (size_t)d * rr, cudaMemcpyDefault, s);
+  if (e == cudaSuccess && rr > 0) e = cudaMemcpyAsync(p->s_b, desc->corr_b_scale, G * rr * 2, cudaMemcpyDefault, s);
+  if (e == cudaSuccess)
+    e = launch_build_layouts(p, t_codes, reinterpret_cast<uint16_t *>(t_scales), reinterpret_cast<int8_t *>(t_u),
+                             reinterpret_cast<int8_t *>(t_a), reinterpret_cast<uint16_t *>(t_sa), s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  free_tmp();
+  if (e != cudaSuccess) return fail(e);
+  *out = p;
+  return ARCHEAD_OK;
+}
+
+void archead_destroy(archead_pack *pack) {
+  if (!pack) return;
+  cudaSetDevice(pack->device);
+  cudaDeviceSynchronize();
+  free_pack(pack);
+}
+
+archead_status archead_forward_path(archead_pack *pack, const void *x, int64_t M, void *logits,
+                                    archead_out_dtype out_dtype, archead_path path, void *stream) {
+  archead_status st = check_forward_args(pack, x, M, logits);
+  if (st != ARCHEAD_OK || M == 0) return st;
+  if (out_dtype != ARCHEAD_OUT_BF16 && out_dtype != ARCHEAD_OUT_FP32) return ARCHEAD_ERR_INVALID_ARG;
+  return run_forward(pack, x, M, logits, out_dtype == ARCHEAD_OUT_FP32, nullptr, nullptr, path,
+                     static_cast<cudaStream_t>(stream));
+}
+
+archead_status archead_forward(archead_pack *pack, const void *x, int64_t M, void *logits,
+                               archead_out_dtype out_dtype, void *stream) {
+  return archead_forward_path(pack, x, M, logits, out_dtype, ARCHEAD_PATH_AUTO, stream);
+}
+
+archead_status archead_forward_ce_path(archead_pack *pack, const void *x, int64_t M, const int32_t *targets,
+                                       float *ce, archead_path path, void *stream) {
+  archead_status st = check_forward_args(pack, x, M, ce);
+  if (st != ARCHEAD_OK || M == 0) return st;
+  if (!targets || !aligned16(targets)) return ARCHEAD_ERR_INVALID_ARG;
+  return run_forward(pack, x, M, nullptr, 0, targets, ce, path, static_cast<cudaStream_t>(stream));
+}
+
+archead_status archead_forward_ce(archead_pack *pack, const void *x, int64_t M, const int32_t *targets, float *ce,
+                                  void *stream) {
+  return archead_forward_ce_path(pack, x, M, targets, ce, ARCHEAD_PATH_AUTO, stream);
+}
+
+archead_status archead_forward_host(archead_pack *pack, const void *x_host, int64_t M, void *logits_host,
+                                    archead_out_dtype out_dtype, void *stream) {
+  if (!pack || M < 0 || !x_host || !logits_host) return ARCHEAD_ERR_INVALID_ARG;
+  if (out_dtype != ARCHEAD_OUT_BF16 && out_dtype != ARCHEAD_OUT_FP32) return ARCHEAD_ERR_INVALID_ARG;
+  if (M == 0) return ARCHEAD_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  AH_CUDA(cudaSetDevice(pack->device));
+  const size_t xb = (size_t)M * pack->d * 2;
+  const size_t yb = (size_t)M * pack->V * (out_dtype == ARCHEAD_OUT_FP32 ? 4 : 2);
+  if (xb > pack->xh_bytes || yb > pack->yh_bytes) {
+    AH_CUDA(cudaStreamSynchronize(s));
+    if (xb > pack->xh_bytes) {
+      if (pack->xh_dev) cudaFree(pack->xh_dev), pack->owned_bytes -= (int64_t)pack->xh_bytes;
+      pack->xh_dev = nullptr;
+      pack->xh_bytes = 0;
+      AH_CUDA(cudaMalloc(&pack->xh_dev, xb));
+      pack->xh_bytes = xb;
+      pack->owned_bytes += (int64_t)xb;
+    }
+    if (yb > pack->yh_bytes) {
+      if (pack->yh_dev) cudaFree(pack->yh_dev), pack->owned_bytes -= (int64_t)pack->yh_bytes;
+      pack->yh_dev = nullptr;
+      pack->yh_bytes = 0;
+      AH_CUDA(cudaMalloc(&pack->yh_dev, yb));
+      pack->yh_bytes = yb;
+      pack->owned_bytes += (int64_t)yb;
+    }
+  }
+  AH_CUDA(cudaMemcpyAsync(pack->xh_dev, x_host, xb, cudaMemcpyHostToDevice, s));
+  archead_status st = archead_forward(pack, pack->xh_dev, M, pack->yh_dev, out_dtype, stream);
+  if (st != ARCHEAD_OK) return st;
+  AH_CUDA(cudaMemcpyAsync(logits_host, pack->yh_dev, yb, cudaMemcpyDeviceToHost, s));
+  AH_CUDA(cudaStreamSynchronize(s));
+  return ARCHEAD_OK;
+}
+
+int64_t archead_pack_bytes(const archead_pack *p) {
+  if (!p) return -1;
+  const int64_t V = p->V, d = p->d, rc = p->rc, rr = p->rr, G = p->G;
+  int64_t b = V * d / 2 + V * G * 2;          // INT4 residual + group scales
+  b += V * rc + rc * 2 + d * rc + rc * 2;     // core factors + column scales
+  b += V * rr + (rr > 0 ? V * 2 : 0);         // correction left + row scales
+  b += d * rr + G * rr * 2;                   // correction right + group scales
+  return b;
+}
+
+int64_t archead_device_bytes(const archead_pack *p) { return p ? p->owned_bytes : -1; }
+
+archead_status archead_debug_dequant(const archead_pack *pack, int component, int64_t row0, int64_t nrows,
+                                     float *out, void *stream) {
+  if (!pack || !out || row0 < 0 || nrows < 0 || component < 0 || component > 4) return ARCHEAD_ERR_INVALID_ARG;
+  const int64_t limit = (component == 2 || component == 4) ? pack->d : pack->V;
+  if (row0 + nrows > limit) return ARCHEAD_ERR_INVALID_ARG;
+  if ((component == 1 || component == 2) && pack->rc == 0) return ARCHEAD_ERR_INVALID_ARG;
+  if ((component == 3 || component == 4) && pack->rr == 0) return ARCHEAD_ERR_INVALID_ARG;
+  AH_CUDA(cudaSetDevice(pack->device));
+  AH_CUDA(launch_debug_dequant(pack, component, row0, nrows, out, static_cast<cudaStream_t>(stream)));
+  return ARCHEAD_OK;
+}
+
+archead_status archead_sync_status(archead_pack *pack, void *stream) {
+  if (!pack) return ARCHEAD_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  AH_CUDA(cudaSetDevice(pack->device));
+  AH_CUDA(cudaStreamSynchronize(s));
+  int word = 0;
+  AH_CUDA(cudaMemcpy(&word, pack->err, sizeof(int), cudaMemcpyDeviceToHost));
+  AH_CUDA(cudaMemset(pack->err, 0, sizeof(int)));
+  if (word & kErrWaitTimeout) return ARCHEAD_ERR_DEVICE_TIMEOUT;
+  if (word & kErrTargetRange) return ARCHEAD_ERR_TARGET_RANGE;
+  return ARCHEAD_OK;
+}
+
+archead_status archead_set_wait_budget(archead_pack *pack, int64_t cycles) {
+  if (!pack || cycles <= 0) return ARCHEAD_ERR_INVALID_ARG;
+  pack->wait_budget = cycles;
+  return ARCHEAD_OK;
+}
+
+archead_status archead_debug_wait_timeout(archead_pack *pack, void *stream) {
+  if (!pack) return ARCHEAD_ERR_INVALID_ARG;
+  AH_CUDA(cudaSetDevice(pack->device));
+  AH_CUDA(launch_wait_timeout_probe(pack->err, pack->wait_budget, static_cast<cudaStream_t>(stream)));
+  return ARCHEAD_OK;
+}
+
+archead_status archead_profile_enable(archead_pack *pack, int enable) {
+  if (!pack) return ARCHEAD_ERR_INVALID_ARG;
+  pack->profiling = enable != 0;
+  return ARCHEAD_OK;
+}
+
+int archead_profile_read(archead_pack *pack, archead_kernel_stat *out, int max_entries) {
+  if (!pack || (!out && max_entries > 0)) return -1;
+  for (auto &t : pack->timers) {
+    for (auto &pr : t.pending) {
+      float ms = 0.f;
+      if (cudaEventSynchronize(pr.second) == cudaSuccess && cudaEventElapsedTime(&ms, pr.first, pr.second) == cudaSuccess) {
+        t.total_ms += ms;
+        t.launches += 1;
+      }
+      cudaEventDestroy(pr.first);
+      cudaEventDestroy(pr.second);
+    }
+    t.pending.clear();
+  }
+  int n = 0;
+  for (auto &t : pack->timers) {
+    if (n >= max_entries) break;
+    out[n].name = t.name;
+    out[n].launches = t.launches;
+    out[n].total_ms = t.total_ms;
+    ++n;
+  }
+  return n;
+}
+
+const char *archead_status_string(archead_status st) {
+  switch (st) {
+    case ARCHEAD_OK: return "ARCHEAD_OK";
+    case ARCHEAD_ERR_INVALID_ARG: return "ARCHEAD_ERR_INVALID_ARG";
+    case ARCHEAD_ERR_UNSUPPORTED: return "ARCHEAD_ERR_UNSUPPORTED";
+    case ARCHEAD_ERR_OOM: return "ARCHEAD_ERR_OOM";
+    case ARCHEAD_ERR_CUDA: return "ARCHEAD_ERR_CUDA";
+    case ARCHEAD_ERR_DEVICE_TIMEOUT: return "ARCHEAD_ERR_DEVICE_TIMEOUT";
+    case ARCHEAD_ERR_TARGET_RANGE: return "ARCHEAD_ERR_TARGET_RANGE";
+  }
+  return "ARCHEAD_ERR_UNKNOWN";
+}
+
+const char *archead_last_error(void) { return g_last_error.c_str(); }
+
+}  // extern "C"

@@ -1,0 +1,138 @@
+// Internal definitions shared by the host API and the kernels of libarchead.
+//
+// Device layouts (all built by archead_pack_create from the canonical layout):
+//
+//  Residual codes, "fragment-native" tiling.  The vocabulary is cut into
+//  tiles of 128 rows (V padded with zero rows), d into chunks of 64.  Chunk
+//  (vt, kc) is 4 KB: [mi 0..7][lane 0..31][word j 0..3] of 32-bit words.
+//  Word j of lane (gq = lane/4, cq = lane%4) in m-tile mi holds the 8 codes an
+//  m16n8k16 A-fragment needs for k16-step 4*kc + j: nibble p (pair i = p%4,
+//  half h = p/4) is row 16*mi + gq + 8*(i%2), column 16*(4*kc+j) + 2*cq +
+//  8*(i/2) + h.  Codes are stored offset-binary (code + 8).
+//    byte offset = ((((vt*KC + kc)*8 + mi)*32 + lane)*4 + j)*4,   KC = d/64
+//
+//  Residual scales: [vt][G][128] fp16 bits (row within tile fastest).
+//
+//  Low-rank codes: the extended rank axis kk in [0, LR) with LR = RCP + RRP,
+//  RCP = r_c rounded up to 32, RRP = r_r rounded up to 32: kk < RCP is
+//  core_u[:, kk], kk >= RCP is corr_a[:, kk - RCP] (zero beyond the rank).
+//  Step ls (16 wide) of tile vt: [mi][lane][8 bytes], bytes 2i, 2i+1 = pair i
+//  (same row/column rule as above with 16*ls in place of the k16 offset),
+//  stored offset-binary (code + 128).
+//    byte offset = (((vt*NLS + ls)*8 + mi)*32 + lane)*8,          NLS = LR/16
+//
+//  Correction row scales: [V_pad] fp16 bits (zero on padding rows).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "archead.h"
+
+namespace archead {
+
+constexpr int kTileRows = 128;     // vocabulary rows per tile
+constexpr int kChunkK = 64;        // d per code chunk
+constexpr int kChunkBytes = 4096;  // 128 rows x 64 codes / 2
+constexpr int kLrStepBytes = 2048; // 128 rows x 16 codes
+constexpr int kDecodeMaxTokens = 16;
+constexpr int kPrepassKSplit = 256;  // d per pre-pass block
+constexpr int64_t kDefaultWaitBudget = 2000000000LL;  // cycles, about one second
+
+struct DecodeParams {
+  const uint8_t *codes;
+  const uint16_t *scales;
+  const uint8_t *lr_codes;
+  const uint16_t *s_a;
+  const uint32_t *xs;   // x fragments for this token chunk
+  const uint32_t *ts;   // t hi/lo fragments for this token chunk
+  int64_t V;
+  int num_tiles, d, G, g, g_shift, nls, nls_core;  // g_shift = log2(g / 16)
+  int M;                // tokens in this chunk (1..16)
+  int m0;               // index of the chunk's first token
+  int NT;               // n-tiles of 8 tokens (1 or 2)
+  void *out;            // logits [M_total][V] (NULL in CE mode)
+  int out_fp32;
+  // CE mode (out == NULL)
+  const int32_t *targets;  // [M_total]
+  float2 *ce_part;         // [num_units][M_total] (max, sum exp)
+  float *ce_tlogit;        // [M_total]
+  int M_total;
+  int *err;
+  int64_t wait_budget;
+};
+
+struct PrepassParams {
+  const uint16_t *x;       // [M][d] bf16
+  const int8_t *q_v;       // [d][r_c]
+  const int8_t *q_b;       // [d][r_r]
+  const uint16_t *s_b;     // [G][r_r]
+  const uint16_t *s_u, *s_v;
+  int M, d, g, rc, rr, rcp, rrp, lr;
+  float *partial;          // [d/256][M][LR]
+  // outputs of finalize
+  uint32_t *ts;            // decode t fragments, per 16-token chunk
+  uint16_t *T;             // prefill extended-K operand [M][2*LR] bf16 (may be NULL)
+  uint32_t *xs;            // decode x fragments, per 16-token chunk (may be NULL)
+};
+
+struct KernelTimer {
+  const char *name;
+  int64_t launches = 0;
+  double total_ms = 0.0;
+  std::vector<std::pair<cudaEvent_t, cudaEvent_t>> pending;
+};
+
+}  // namespace archead
+
+struct archead_pack {
+  int device = 0;
+  int sm_count = 0;
+  int64_t V = 0, V_pad = 0;
+  int d = 0, rc = 0, rr = 0, g = 0, G = 0, rcp = 0, rrp = 0, lr = 0, nls = 0, nls_core = 0;
+  int num_tiles = 0;
+  // device buffers owned by the pack
+  uint8_t *codes = nullptr;
+  uint16_t *scales = nullptr;
+  uint8_t *lr_codes = nullptr;
+  uint16_t *s_a = nullptr;
+  int8_t *q_v = nullptr, *q_b = nullptr;
+  uint16_t *s_u = nullptr, *s_v = nullptr, *s_b = nullptr;
+  int *err = nullptr;
+  int64_t owned_bytes = 0;
+  // workspace (grown on demand)
+  void *ws = nullptr;
+  size_t ws_bytes = 0;
+  // host staging for archead_forward_host
+  void *xh_dev = nullptr, *yh_dev = nullptr;
+  size_t xh_bytes = 0, yh_bytes = 0;
+  int64_t wait_budget = archead::kDefaultWaitBudget;
+  bool profiling = false;
+  std::vector<archead::KernelTimer> timers;
+};
+
+namespace archead {
+
+// Kernel launchers (each returns the launch's cudaError_t).
+cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, const uint16_t *res_scales,
+                                 const int8_t *core_u, const int8_t *corr_a, const uint16_t *corr_a_scale,
+                                 cudaStream_t s);
+cudaError_t launch_debug_dequant(const archead_pack *p, int comp, int64_t row0, int64_t nrows, float *out,
+                                 cudaStream_t s);
+cudaError_t launch_prepass(const PrepassParams &pp, cudaStream_t s, archead_pack *p);
+cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s);
+int decode_num_units(const archead_pack *p);
+int decode_parts_per_unit();
+bool decode_supported(int d, int nls);
+cudaError_t launch_ce_finalize(const float2 *part, int num_parts, const float *tlogit, const int32_t *targets,
+                               int64_t V, int M, float *ce, int *err, cudaStream_t s);
+cudaError_t launch_wait_timeout_probe(int *err, int64_t budget, cudaStream_t s);
+
+// Profiling hooks (no-ops unless profiling is enabled on the pack).
+void timer_begin(archead_pack *p, const char *name, cudaStream_t s, cudaEvent_t *ev0);
+void timer_end(archead_pack *p, const char *name, cudaStream_t s, cudaEvent_t ev0);
+
+}  // namespace archead

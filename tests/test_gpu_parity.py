@@ -1,0 +1,174 @@
+"""CUDA path vs the fp64 oracle on small heads (several tiles, ragged tails,
+every supported group size, rank 0 branches), through the C ABI."""
+
+import zlib
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_02703_gb300 import archead
+from synth import HeadShape, make_head, make_hidden, make_targets
+from tests import gpu_util as gu
+
+pytestmark = pytest.mark.gpu
+
+SHAPES = {
+    "ragged": HeadShape(V=1000, d=256, core_rank=16, corr_rank=8, group_size=64),
+    "tiny": HeadShape(V=4096, d=512, core_rank=64, corr_rank=16, group_size=64),
+    "g32": HeadShape(V=700, d=512, core_rank=24, corr_rank=40, group_size=32),
+    "g128": HeadShape(V=513, d=512, core_rank=128, corr_rank=32, group_size=128),
+    "g256": HeadShape(V=300, d=768, core_rank=8, corr_rank=8, group_size=256),
+    "d320": HeadShape(V=333, d=320, core_rank=5, corr_rank=3, group_size=64),
+    "group_int4": HeadShape(V=640, d=256, core_rank=0, corr_rank=0, group_size=64),
+    "core_only": HeadShape(V=640, d=256, core_rank=32, corr_rank=0, group_size=64),
+    "corr_only": HeadShape(V=640, d=256, core_rank=0, corr_rank=32, group_size=64),
+    "max_rank": HeadShape(V=384, d=256, core_rank=256, corr_rank=256, group_size=64),
+    "one_row": HeadShape(V=1, d=64, core_rank=4, corr_rank=4, group_size=32),
+}
+
+_packs = {}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _build():
+    from paper_2608_02703_gb300.build import build
+
+    build()
+    yield
+    for p, _ in _packs.values():
+        p.close()
+    _packs.clear()
+
+
+def get(name):
+    if name not in _packs:
+        shape = SHAPES[name]
+        head = make_head(shape, seed=zlib.crc32(name.encode()) % 1000)
+        _packs[name] = (archead.archead_pack_create(head, shape), head)
+    return _packs[name]
+
+
+@pytest.mark.parametrize("name", sorted(SHAPES))
+def test_dequant_bit_exact(name):
+    import torch
+
+    pack, head = get(name)
+    shape = SHAPES[name]
+    comps = [("residual", shape.V, shape.d)]
+    if shape.core_rank:
+        comps += [("core_u", shape.V, shape.core_rank), ("core_v", shape.d, shape.core_rank)]
+    if shape.corr_rank:
+        comps += [("corr_a", shape.V, shape.corr_rank), ("corr_b", shape.d, shape.corr_rank)]
+    for comp, rows, cols in comps:
+        out = torch.full((rows, cols), float("nan"), dtype=torch.float32, device="cuda")
+        archead.archead_debug_dequant(pack, comp, 0, rows, out)
+        torch.cuda.synchronize()
+        got = out.cpu().numpy()
+        ref = oracle.component(head, shape, comp)
+        assert np.array_equal(got.astype(np.float64), ref), f"{name}/{comp} not bit-exact"
+        assert np.array_equal(got.view(np.uint32), ref.astype(np.float32).view(np.uint32))
+
+
+@pytest.mark.parametrize("name", sorted(SHAPES))
+@pytest.mark.parametrize("M", [1, 3, 8, 9, 16])
+def test_decode_logits(name, M):
+    pack, head = get(name)
+    shape = SHAPES[name]
+    x = make_hidden(shape.d, M, seed=M, n_outliers=shape.n_outliers)
+    ref = oracle.logits(head, shape, x)
+    got = gu.forward(pack, x, archead.OUT_FP32, archead.PATH_DECODE)
+    gu.check_logits(got, ref, where=f"{name} M={M} fp32")
+    gu.check_argmax(got, ref, where=f"{name} M={M}")
+    got16 = gu.forward(pack, x, archead.OUT_BF16, archead.PATH_DECODE)
+    gu.check_logits(got16, ref, bf16=True, where=f"{name} M={M} bf16")
+
+
+@pytest.mark.parametrize("name", ["ragged", "tiny", "g32", "max_rank"])
+@pytest.mark.parametrize("M", [17, 40, 133])
+def test_logits_many_tokens(name, M):
+    pack, head = get(name)
+    shape = SHAPES[name]
+    x = make_hidden(shape.d, M, seed=M)
+    ref = oracle.logits(head, shape, x)
+    for path in (archead.PATH_AUTO, archead.PATH_DECODE, archead.PATH_PREFILL):
+        got = gu.forward(pack, x, archead.OUT_FP32, path)
+        gu.check_logits(got, ref, where=f"{name} M={M} path={path}")
+        gu.check_argmax(got, ref, where=f"{name} M={M} path={path}")
+
+
+@pytest.mark.parametrize("name", ["ragged", "tiny", "g32", "g256", "corr_only", "one_row"])
+@pytest.mark.parametrize("M", [1, 5, 16, 33])
+def test_cross_entropy(name, M):
+    pack, head = get(name)
+    shape = SHAPES[name]
+    x = make_hidden(shape.d, M, seed=100 + M)
+    t = make_targets(shape.V, M, seed=M)
+    ref = oracle.cross_entropy(head, shape, x, t)["ce"]
+    for path in (archead.PATH_AUTO, archead.PATH_DECODE, archead.PATH_PREFILL):
+        got, st = gu.forward_ce(pack, x, t, path)
+        assert st == archead.OK
+        err = np.abs(got - ref)
+        assert np.all(err <= gu.CE_ABS), f"{name} M={M} path={path}: max|dCE|={err.max():.3e}"
+
+
+def test_ce_target_out_of_range():
+    pack, head = get("ragged")
+    shape = SHAPES["ragged"]
+    x = make_hidden(shape.d, 4, seed=3)
+    t = np.array([5, shape.V, -1, 7], dtype=np.int32)
+    got, st = gu.forward_ce(pack, x, t)
+    assert st == archead.ERR_TARGET_RANGE
+    assert np.isnan(got[1]) and np.isnan(got[2])
+    ref = oracle.cross_entropy(head, shape, x[[0, 3]], t[[0, 3]])["ce"]
+    assert np.all(np.abs(got[[0, 3]] - ref) <= gu.CE_ABS)
+    assert archead.archead_sync_status(pack) == archead.OK  # the error word was cleared
+
+
+def test_zero_tokens_is_a_no_op():
+    import torch
+
+    pack, _ = get("ragged")
+    y = torch.zeros((1, 1), dtype=torch.float32, device="cuda")
+    archead.archead_forward(pack, y, 0, y, archead.OUT_FP32)
+    assert archead.archead_sync_status(pack) == archead.OK
+
+
+def test_forward_host_matches_device():
+    import torch
+
+    pack, head = get("tiny")
+    shape = SHAPES["tiny"]
+    x = make_hidden(shape.d, 4, seed=9)
+    dev = gu.forward(pack, x, archead.OUT_BF16)
+    xh = torch.from_numpy(x.view(np.int16)).pin_memory()
+    yh = torch.empty((4, shape.V), dtype=torch.bfloat16).pin_memory()
+    archead.archead_forward_host(pack, xh, 4, yh, archead.OUT_BF16)
+    assert np.array_equal(yh.float().numpy().astype(np.float64), dev)
+
+
+def test_wait_timeout_is_reported_and_recoverable():
+    pack, head = get("ragged")
+    archead.archead_set_wait_budget(pack, 20_000)  # cycles: a few microseconds
+    archead.archead_debug_wait_timeout(pack)
+    assert archead.archead_sync_status(pack) == archead.ERR_DEVICE_TIMEOUT
+    archead.archead_set_wait_budget(pack, 2_000_000_000)
+    shape = SHAPES["ragged"]
+    x = make_hidden(shape.d, 2, seed=1)
+    gu.check_logits(gu.forward(pack, x), oracle.logits(head, shape, x), where="after timeout")
+
+
+def test_pack_bytes_follow_eq10():
+    for name in ("tiny", "group_int4", "core_only", "max_rank"):
+        pack, head = get(name)
+        assert archead.archead_pack_bytes(pack) == oracle.packed_bytes(SHAPES[name])
+        assert archead.archead_device_bytes(pack) >= archead.archead_pack_bytes(pack)
+
+
+def test_deterministic():
+    pack, _ = get("tiny")
+    shape = SHAPES["tiny"]
+    x = make_hidden(shape.d, 16, seed=4)
+    a = gu.forward(pack, x)
+    b = gu.forward(pack, x)
+    assert np.array_equal(a, b)
