@@ -42,7 +42,7 @@ cudaError_t dev_alloc(archead_pack *p, T **ptr, size_t bytes) {
 void free_pack(archead_pack *p) {
   if (!p) return;
   void *bufs[] = {p->codes, p->scales, p->lr_codes, p->s_a, p->q_v, p->q_b, p->s_u,
-                  p->s_v,   p->s_b,    p->err,      p->ws,  p->xh_dev, p->yh_dev};
+                  p->s_v,   p->s_b,    p->err,      p->ws,  p->xh_dev, p->yh_dev, p->counters};
   for (void *b : bufs)
     if (b) cudaFree(b);
   for (auto &t : p->timers)
@@ -81,9 +81,30 @@ cudaError_t ensure_workspace(archead_pack *p, size_t bytes, cudaStream_t s) {
   return cudaSuccess;
 }
 
+// Block counters of the pre-pass: zeroed once when (re)allocated; every
+// pre-pass call leaves them zero again.
+cudaError_t ensure_counters(archead_pack *p, int n, cudaStream_t s) {
+  if (n <= p->counters_len) return cudaSuccess;
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return e;
+  if (p->counters) {
+    cudaFree(p->counters);
+    p->owned_bytes -= (int64_t)p->counters_len * 4;
+    p->counters = nullptr;
+    p->counters_len = 0;
+  }
+  const int len = std::max(n, 1024);
+  e = cudaMalloc(&p->counters, (size_t)len * 4);
+  if (e != cudaSuccess) return e;
+  e = cudaMemset(p->counters, 0, (size_t)len * 4);
+  if (e != cudaSuccess) return e;
+  p->counters_len = len;
+  p->owned_bytes += (int64_t)len * 4;
+  return cudaSuccess;
+}
+
 struct ForwardPlan {
-  PrepassParams pp{};
-  size_t ce_part_off = 0, tlogit_off = 0, total = 0;
+  size_t partial_off = 0, ts_off = 0, ce_part_off = 0, tlogit_off = 0, total = 0;
   int nchunks = 0;
 };
 
@@ -91,25 +112,20 @@ struct ForwardPlan {
 ForwardPlan plan_decode(archead_pack *p, int64_t M, bool ce) {
   ForwardPlan f;
   Carve c;
-  const int nsplit = (p->d + kPrepassKSplit - 1) / kPrepassKSplit;
   f.nchunks = (int)((M + kDecodeMaxTokens - 1) / kDecodeMaxTokens);
-  size_t partial = c.take((size_t)nsplit * M * std::max(p->lr, 1) * sizeof(float));
-  size_t ts = c.take((size_t)f.nchunks * std::max(p->nls, 1) * 1024);
-  size_t xs = c.take((size_t)f.nchunks * 32 * p->d);
+  f.partial_off = c.take(prepass_partial_bytes((int)M, p->lr, p->d));
+  f.ts_off = c.take((size_t)f.nchunks * std::max(p->nls, 1) * 1024);
   if (ce) {
     f.ce_part_off = c.take((size_t)decode_num_units(p) * decode_parts_per_unit() * M * sizeof(float2));
     f.tlogit_off = c.take((size_t)M * sizeof(float));
   }
   f.total = c.off;
-  f.pp.partial = reinterpret_cast<float *>(partial);  // offsets; rebased once the workspace exists
-  f.pp.ts = reinterpret_cast<uint32_t *>(ts);
-  f.pp.xs = reinterpret_cast<uint32_t *>(xs);
   return f;
 }
 
 template <typename T>
-T *rebase(void *base, T *off) {
-  return reinterpret_cast<T *>(static_cast<char *>(base) + reinterpret_cast<uintptr_t>(off));
+T *at(void *base, size_t off) {
+  return reinterpret_cast<T *>(static_cast<char *>(base) + off);
 }
 
 archead_status check_forward_args(archead_pack *p, const void *x, int64_t M, const void *out) {
@@ -120,13 +136,7 @@ archead_status check_forward_args(archead_pack *p, const void *x, int64_t M, con
   return ARCHEAD_OK;
 }
 
-// Decode path over M tokens, 16 at a time.  out == nullptr selects CE mode.
-archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
-                          const int32_t *targets, float *ce, cudaStream_t s) {
-  if (!decode_supported(p->d, p->nls)) return ARCHEAD_ERR_UNSUPPORTED;
-  const bool ce_mode = out == nullptr;
-  ForwardPlan f = plan_decode(p, M, ce_mode);
-  AH_CUDA(ensure_workspace(p, f.total, s));
+PrepassParams prepass_params(archead_pack *p, const void *x, int64_t M) {
   PrepassParams pp{};
   pp.x = static_cast<const uint16_t *>(x);
   pp.q_v = p->q_v;
@@ -142,9 +152,21 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   pp.rcp = p->rcp;
   pp.rrp = p->rrp;
   pp.lr = p->lr;
-  pp.partial = rebase(p->ws, f.pp.partial);
-  pp.ts = rebase(p->ws, f.pp.ts);
-  pp.xs = rebase(p->ws, f.pp.xs);
+  return pp;
+}
+
+// Decode path over M tokens, 16 at a time.  out == nullptr selects CE mode.
+archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
+                          const int32_t *targets, float *ce, cudaStream_t s) {
+  if (!decode_supported(p->d_pad, p->nls, p->g)) return ARCHEAD_ERR_UNSUPPORTED;
+  const bool ce_mode = out == nullptr;
+  ForwardPlan f = plan_decode(p, M, ce_mode);
+  AH_CUDA(ensure_workspace(p, f.total, s));
+  AH_CUDA(ensure_counters(p, prepass_pairs((int)M, p->lr), s));
+  PrepassParams pp = prepass_params(p, x, M);
+  pp.partial = at<float>(p->ws, f.partial_off);
+  pp.counters = p->counters;
+  pp.ts = at<uint32_t>(p->ws, f.ts_off);
   pp.T = nullptr;
   AH_CUDA(launch_prepass(pp, s, p));
 
@@ -153,20 +175,20 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   dp.scales = p->scales;
   dp.lr_codes = p->lr_codes;
   dp.s_a = p->s_a;
+  dp.x = static_cast<const uint16_t *>(x);
   dp.V = p->V;
   dp.num_tiles = p->num_tiles;
   dp.d = p->d;
-  dp.G = p->G;
+  dp.d_pad = p->d_pad;
+  dp.G_pad = p->G_pad;
   dp.g = p->g;
-  dp.g_shift = 0;
-  while ((16 << dp.g_shift) < p->g) ++dp.g_shift;
   dp.nls = p->nls;
   dp.nls_core = p->nls_core;
   dp.out = out;
   dp.out_fp32 = out_fp32;
   dp.targets = targets;
-  dp.ce_part = ce_mode ? rebase(p->ws, reinterpret_cast<float2 *>(f.ce_part_off)) : nullptr;
-  dp.ce_tlogit = ce_mode ? rebase(p->ws, reinterpret_cast<float *>(f.tlogit_off)) : nullptr;
+  dp.ce_part = ce_mode ? at<float2>(p->ws, f.ce_part_off) : nullptr;
+  dp.ce_tlogit = ce_mode ? at<float>(p->ws, f.tlogit_off) : nullptr;
   dp.M_total = (int)M;
   dp.err = p->err;
   dp.wait_budget = p->wait_budget;
@@ -175,11 +197,12 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
     dp.m0 = c * kDecodeMaxTokens;
     dp.M = (int)std::min<int64_t>(kDecodeMaxTokens, M - dp.m0);
     dp.NT = dp.M > 8 ? 2 : 1;
-    dp.xs = pp.xs + (size_t)c * 8 * p->d;
     dp.ts = pp.ts + (size_t)c * p->nls * 256;
     cudaEvent_t ev = nullptr;
     timer_begin(p, "decode", s, &ev);
-    cudaError_t e = launch_decode(dp, grid, s);
+    // The first chunk overlaps the pre-pass grid (programmatic dependent launch).
+    const bool pdl = c == 0 && p->lr > 0 && !p->profiling;
+    cudaError_t e = launch_decode(dp, grid, s, pdl);
     timer_end(p, "decode", s, ev);
     if (e != cudaSuccess) return cuda_status(e);
   }
@@ -275,6 +298,8 @@ archead_status archead_pack_create(const archead_desc *desc, void *stream, arche
   p->rr = rr;
   p->g = g;
   p->G = (int)(d / g);
+  p->d_pad = (int)round_up(d, 128);
+  p->G_pad = p->d_pad / g;
   p->num_tiles = (int)((V + kTileRows - 1) / kTileRows);
   p->V_pad = (int64_t)p->num_tiles * kTileRows;
   p->rcp = (int)round_up(rc, 32);
@@ -284,8 +309,8 @@ archead_status archead_pack_create(const archead_desc *desc, void *stream, arche
   p->nls_core = p->rcp / 16;
 
   const size_t G = p->G;
-  if ((e = dev_alloc(p, &p->codes, (size_t)p->V_pad * d / 2)) != cudaSuccess) return fail(e);
-  if ((e = dev_alloc(p, &p->scales, (size_t)p->V_pad * G * 2)) != cudaSuccess) return fail(e);
+  if ((e = dev_alloc(p, &p->codes, (size_t)p->V_pad * p->d_pad / 2)) != cudaSuccess) return fail(e);
+  if ((e = dev_alloc(p, &p->scales, (size_t)p->V_pad * p->G_pad * 2)) != cudaSuccess) return fail(e);
   if ((e = dev_alloc(p, &p->lr_codes, (size_t)p->num_tiles * p->nls * kLrStepBytes)) != cudaSuccess) return fail(e);
   if ((e = dev_alloc(p, &p->s_a, (size_t)p->V_pad * 2)) != cudaSuccess) return fail(e);
   if ((e = dev_alloc(p, &p->q_v, (size_t)d * rc)) != cudaSuccess) return fail(e);

@@ -1,124 +1,198 @@
 // Memory-bound decode kernel (M <= 16 tokens) of the packed LM-head forward
-// (paper, Section 3.2, Eq. 7; Appendix B "At inference ... core path and
-// correction path separately").
+// (paper, Section 3.2, Eq. 7; Appendix B: the core and correction paths are
+// evaluated separately and no dense head is formed).
 //
-// Persistent grid, one block per SM.  A unit of work is 256 vocabulary rows
-// (two 128-row tiles).  One producer warp streams each unit's INT4 codes,
+// Persistent grid, one block per SM.  A unit of work is 512 vocabulary rows
+// (four 128-row tiles).  One producer warp streams each unit's INT4 codes,
 // group scales and low-rank codes with 1-D bulk TMA copies into a ring of
-// shared-memory stages (mbarrier full/empty pairs).  Eight consumer warps each
-// own two 16-row m-tiles.  Per 16-wide k step a consumer converts one 32-bit
+// shared-memory stages (mbarrier full/empty pairs).  Sixteen consumer warps each
+// own two 16-row m-tiles.  Per 16-wide k step a consumer turns one 32-bit
 // word of offset-binary nibbles into the four bf16 A-fragment registers of an
-// m16n8k16 MMA (exact small integers) and multiplies them with the bf16
-// hidden states (B fragments, tokens on the 8-wide side) held in shared
-// memory, accumulating in fp32.  At the end of every quantisation group the
+// m16n8k16 MMA (exact small integers) and multiplies them with the bf16 hidden
+// states (B fragments, tokens on the 8-wide side, staged once per block by
+// TMA), accumulating in fp32.  At the end of every quantisation group the
 // partial sums are promoted by that row's group scale in fp32.  The rank-r
 // branches follow as extra k steps: int8 codes of A_c (core) or A_w
-// (correction) times the bf16 hi/lo split of t = x V (pre-pass), the
-// correction promoted by the row scale of A_w.
+// (correction) times the bf16 hi/lo split of t = x V from the pre-pass, the
+// correction promoted by the row scale of A_w.  The pre-pass runs as the
+// preceding grid; this kernel starts streaming under programmatic dependent
+// launch and waits for the pre-pass only before the first rank-r stage.
 #include "device.cuh"
 #include "internal.h"
 
 namespace archead {
 
-constexpr int kDecConsumerWarps = 8;
-constexpr int kDecThreads = (kDecConsumerWarps + 1) * 32;
-constexpr int kDecStageCodeBytes = 2 * 2 * kChunkBytes;  // 2 tiles x 2 chunks (128 of d)
-constexpr int kDecStageScaleBytes = 2 * 4 * kTileRows * 2;  // 2 tiles x up to 4 groups
-constexpr int kDecStageBytes = kDecStageCodeBytes + kDecStageScaleBytes;
-constexpr int kDecLrStepsPerStage = 4;
+constexpr int kDecWarps = 8;                      // consumer warps
+constexpr int kDecThreads = (kDecWarps + 1) * 32; // + producer warp
+constexpr int kDecTiles = 4;                      // 128-row tiles per unit
+constexpr int kDecMT = 4;                         // m-tiles per consumer warp (2 warps per tile)
 constexpr int kSmemLimit = 227 * 1024;
 
-struct DecodeSmemPlan {
-  int stages;
-  size_t xs_off, ts_off, bar_off, total;
+// 64-wide chunks of d per ring stage, by number of 8-token n-tiles.  The
+// shared-memory plan and the kernel instance launched both take it from here.
+__host__ __device__ constexpr int stage_chunks(int NT) { return NT == 1 ? 2 : 1; }
+
+// Stage geometry for SC chunks (64 of d each) per stage.
+template <int SC>
+struct StageGeom {
+  static constexpr int kCodeBytes = kDecTiles * SC * kChunkBytes;  // also holds 2*SC low-rank steps per tile
+  static constexpr int kScaleBytesPerTile = (SC * kChunkK / 32) * kTileRows * 2;  // up to SC*64/g groups (g >= 32)
+  static constexpr int kBytes = kCodeBytes + kDecTiles * kScaleBytesPerTile;
+  static constexpr int kLrSteps = 2 * SC;  // 16-wide low-rank steps per stage (2 KB per tile each)
 };
 
-static DecodeSmemPlan decode_plan(int d, int nls, int NT) {
-  DecodeSmemPlan pl{};
-  const size_t xs_bytes = (size_t)NT * 16 * d;
+struct DecodePlan {
+  int stages, sc;
+  size_t xs_off, ts_off, xsum_off, bar_off, total;
+};
+
+__host__ __device__ __forceinline__ int xs_row_elems(int d_pad) { return d_pad + 8; }  // +16 B: rows on distinct banks
+
+// Shared memory: the stage ring, M rows of hidden states, the rank-r
+// fragments, the per-group sums of x, and the barriers.  The total leaves
+// room for one pre-pass block on the same SM (programmatic dependent launch
+// overlaps the two grids) whenever the stage ring still holds 96 KB.
+static DecodePlan decode_plan(int d_pad, int nls, int g, int M) {
+  DecodePlan pl{};
+  pl.sc = stage_chunks(M > 8 ? 2 : 1);
+  const size_t stage_bytes = pl.sc == 2 ? StageGeom<2>::kBytes : StageGeom<1>::kBytes;
+  const size_t xs_bytes = (size_t)M * xs_row_elems(d_pad) * 2;
   const size_t ts_bytes = (size_t)nls * 1024;
-  const size_t fixed = xs_bytes + ts_bytes + 256;
-  int st = 4;
-  while (st >= 2 && fixed + (size_t)st * kDecStageBytes > (size_t)kSmemLimit) --st;
+  const size_t xsum_bytes = (size_t)(d_pad / g) * kDecodeMaxTokens * 4;
+  const size_t fixed = xs_bytes + ts_bytes + xsum_bytes + 256;
+  const size_t shared_cap = (size_t)kSmemLimit - prepass_smem(M) - 2048;
+  int st = 8;
+  while (st >= 2 && fixed + (size_t)st * stage_bytes > shared_cap) --st;
+  if (st < 2 || (size_t)st * stage_bytes < 96 * 1024) {  // too shallow a ring: give up co-residency
+    st = 8;
+    while (st >= 2 && fixed + (size_t)st * stage_bytes > (size_t)kSmemLimit) --st;
+  }
   pl.stages = st;
-  pl.xs_off = (size_t)st * kDecStageBytes;
+  pl.xs_off = (size_t)st * stage_bytes;
   pl.ts_off = pl.xs_off + xs_bytes;
-  pl.bar_off = pl.ts_off + ts_bytes;
+  pl.xsum_off = pl.ts_off + ts_bytes;
+  pl.bar_off = pl.xsum_off + xsum_bytes;
   pl.total = pl.bar_off + 256;
   return pl;
 }
 
+// Residual group promotion with the operand bias removed:
+// acc += s_row * (part + nb_tok), nb = -136 * sum of x over the group; part = 0.
+// Residual group promotion with the operand bias removed:
+// acc += s_row * (part + nb_tok), nb = -136 * sum of x over the group.
 template <int NT>
+__device__ __forceinline__ void promote_res(float (&acc)[NT][4], const float (&part)[NT][4], float s_lo, float s_hi,
+                                            const float2 (&nb)[NT]) {
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+    acc[nt][0] = fmaf(s_lo, part[nt][0] + nb[nt].x, acc[nt][0]);
+    acc[nt][1] = fmaf(s_lo, part[nt][1] + nb[nt].y, acc[nt][1]);
+    acc[nt][2] = fmaf(s_hi, part[nt][2] + nb[nt].x, acc[nt][2]);
+    acc[nt][3] = fmaf(s_hi, part[nt][3] + nb[nt].y, acc[nt][3]);
+  }
+}
+
+// acc += f_lo * part (rows gq) and f_hi * part (rows gq + 8).
+template <int NT>
+__device__ __forceinline__ void promote(float (&acc)[NT][4], const float (&part)[NT][4], float f_lo, float f_hi) {
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+    acc[nt][0] = fmaf(f_lo, part[nt][0], acc[nt][0]);
+    acc[nt][1] = fmaf(f_lo, part[nt][1], acc[nt][1]);
+    acc[nt][2] = fmaf(f_hi, part[nt][2], acc[nt][2]);
+    acc[nt][3] = fmaf(f_hi, part[nt][3], acc[nt][3]);
+  }
+}
+
+// NT: n-tiles of 8 tokens; SC: 64-wide chunks per stage; GS: 16-wide k steps per group.
+template <int NT, int SC, int GS>
 __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, int stages, int xs_off, int ts_off,
-                                                                int bar_off) {
+                                                                int xsum_off, int bar_off) {
+  using Geom = StageGeom<SC>;
+  constexpr int SS = 4 * SC;  // 16-wide k steps per stage
   extern __shared__ __align__(1024) uint8_t smem[];
-  uint8_t *stage_base = smem;
-  const uint32_t *xs_s = reinterpret_cast<const uint32_t *>(smem + xs_off);
+  const uint16_t *xs_s = reinterpret_cast<const uint16_t *>(smem + xs_off);
   const uint32_t *ts_s = reinterpret_cast<const uint32_t *>(smem + ts_off);
+  float *xsum_s = reinterpret_cast<float *>(smem + xsum_off);  // [group][16 tokens]: -136 * sum of x
   uint64_t *full = reinterpret_cast<uint64_t *>(smem + bar_off);
-  uint64_t *empty = full + 4;
-  uint64_t *xbar = full + 8;
-  volatile int *abort_flag = reinterpret_cast<volatile int *>(full + 9);
+  uint64_t *empty = full + 8;
+  uint64_t *xbar = full + 16;
+  uint64_t *tbar = full + 17;
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(full + 18);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int KC = p.d / kChunkK;
-  const int res_stages = (KC + 1) / 2;
-  const int lr_stages = (p.nls + kDecLrStepsPerStage - 1) / kDecLrStepsPerStage;
-  const int num_units = (p.num_tiles + 1) / 2;
+  const int KC = p.d_pad / kChunkK;
+  const int res_stages = KC / SC;
+  const int lr_stages = (p.nls + Geom::kLrSteps - 1) / Geom::kLrSteps;
+  const int num_units = (p.num_tiles + kDecTiles - 1) / kDecTiles;
+  const int xrow = xs_row_elems(p.d_pad);
 
+  // Columns [d, d_pad) of the hidden states meet zero codes; zero them so
+  // that no stale pattern (a NaN) reaches the accumulators.
+  if (p.d < p.d_pad) {
+    const int per_row = (p.d_pad - p.d) / 8;  // uint4 per row
+    for (int e = threadIdx.x; e < p.M * per_row; e += blockDim.x) {
+      uint4 *dst = reinterpret_cast<uint4 *>(smem + xs_off + (size_t)(e / per_row) * xrow * 2 + (size_t)p.d * 2);
+      dst[e % per_row] = make_uint4(0, 0, 0, 0);
+    }
+  }
   if (threadIdx.x == 0) {
     for (int i = 0; i < stages; ++i) {
       mbar_init(&full[i], 1);
-      mbar_init(&empty[i], kDecConsumerWarps);
+      mbar_init(&empty[i], kDecWarps);
     }
     mbar_init(xbar, 1);
+    mbar_init(tbar, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
   __syncthreads();
 
-  if (warp == kDecConsumerWarps) {
+  if (warp == kDecWarps) {
     // ---------------- producer warp ----------------
     if (lane != 0) return;
-    const uint32_t xs_bytes = (uint32_t)(NT * 16 * p.d);
-    const uint32_t ts_bytes = (uint32_t)(p.nls * 1024);
-    mbar_arrive_expect_tx(xbar, xs_bytes + ts_bytes);
-    bulk_g2s(smem + xs_off, p.xs, xs_bytes, xbar);
-    if (ts_bytes) bulk_g2s(smem + ts_off, p.ts, ts_bytes, xbar);
+    mbar_arrive_expect_tx(xbar, (uint32_t)(p.M * p.d * 2));
+    for (int m = 0; m < p.M; ++m)
+      bulk_g2s(smem + xs_off + (size_t)m * xrow * 2, p.x + (size_t)(p.m0 + m) * p.d, (uint32_t)(p.d * 2), xbar);
+    bool t_loaded = false;
     int it = 0;
     for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x) {
-      const int ntile = min(2, p.num_tiles - 2 * unit);
+      const int ntile = min(kDecTiles, p.num_tiles - kDecTiles * unit);
       for (int s = 0; s < res_stages + lr_stages; ++s, ++it) {
         const int st = it % stages;
-        const uint32_t ph = (it / stages) & 1;
-        if (!mbar_wait(&empty[st], ph ^ 1, p.wait_budget, abort_flag, p.err)) goto producer_abort;
-        uint8_t *buf = stage_base + (size_t)st * kDecStageBytes;
+        if (s == res_stages && !t_loaded) {
+          // The rank-r fragments come from the pre-pass grid.
+          asm volatile("griddepcontrol.wait;\n" ::: "memory");
+          mbar_arrive_expect_tx(tbar, (uint32_t)(p.nls * 1024));
+          bulk_g2s(smem + ts_off, p.ts, (uint32_t)(p.nls * 1024), tbar);
+          t_loaded = true;
+        }
+        if (!mbar_wait(&empty[st], ((it / stages) & 1) ^ 1, p.wait_budget, abort_flag, p.err)) goto producer_abort;
+        uint8_t *buf = smem + (size_t)st * Geom::kBytes;
         if (s < res_stages) {
-          const int kc0 = 2 * s;
-          const int nkc = min(2, KC - kc0);
+          const int kc0 = s * SC;
           const int g0 = (kc0 * kChunkK) / p.g;
-          const int g1 = ((kc0 + nkc) * kChunkK - 1) / p.g;
+          const int g1 = ((kc0 + SC) * kChunkK - 1) / p.g;
           const int ng = g1 - g0 + 1;
-          mbar_arrive_expect_tx(&full[st], (uint32_t)(ntile * (nkc * kChunkBytes + ng * kTileRows * 2)));
+          mbar_arrive_expect_tx(&full[st], (uint32_t)(ntile * (SC * kChunkBytes + ng * kTileRows * 2)));
           for (int t = 0; t < ntile; ++t) {
-            const int64_t vt = 2 * (int64_t)unit + t;
-            bulk_g2s(buf + t * 2 * kChunkBytes, p.codes + (vt * KC + kc0) * kChunkBytes, nkc * kChunkBytes,
-                     &full[st]);
-            bulk_g2s(buf + kDecStageCodeBytes + t * 4 * kTileRows * 2, p.scales + (vt * p.G + g0) * kTileRows,
+            const int64_t vt = (int64_t)kDecTiles * unit + t;
+            bulk_g2s(buf + t * SC * kChunkBytes, p.codes + (vt * KC + kc0) * kChunkBytes, SC * kChunkBytes, &full[st]);
+            bulk_g2s(buf + Geom::kCodeBytes + t * Geom::kScaleBytesPerTile, p.scales + (vt * p.G_pad + g0) * kTileRows,
                      ng * kTileRows * 2, &full[st]);
           }
         } else {
-          const int ls0 = (s - res_stages) * kDecLrStepsPerStage;
-          const int nl = min(kDecLrStepsPerStage, p.nls - ls0);
+          const int ls0 = (s - res_stages) * Geom::kLrSteps;
+          const int nl = min(Geom::kLrSteps, p.nls - ls0);
           const bool last = (s == res_stages + lr_stages - 1);
           mbar_arrive_expect_tx(&full[st], (uint32_t)(ntile * (nl * kLrStepBytes + (last ? kTileRows * 2 : 0))));
           for (int t = 0; t < ntile; ++t) {
-            const int64_t vt = 2 * (int64_t)unit + t;
-            bulk_g2s(buf + t * kDecLrStepsPerStage * kLrStepBytes, p.lr_codes + (vt * p.nls + ls0) * kLrStepBytes,
+            const int64_t vt = (int64_t)kDecTiles * unit + t;
+            bulk_g2s(buf + t * Geom::kLrSteps * kLrStepBytes, p.lr_codes + (vt * p.nls + ls0) * kLrStepBytes,
                      nl * kLrStepBytes, &full[st]);
             if (last)
-              bulk_g2s(buf + kDecStageCodeBytes + t * kTileRows * 2, p.s_a + vt * kTileRows, kTileRows * 2,
+              bulk_g2s(buf + Geom::kCodeBytes + t * Geom::kScaleBytesPerTile, p.s_a + vt * kTileRows, kTileRows * 2,
                        &full[st]);
           }
         }
@@ -131,150 +205,216 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
       const int j = it - k;
       mbar_wait(&full[j % stages], (j / stages) & 1, p.wait_budget, nullptr, p.err);
     }
+    mbar_wait(xbar, 0, p.wait_budget, nullptr, p.err);
+    if (t_loaded) mbar_wait(tbar, 0, p.wait_budget, nullptr, p.err);
     return;
   }
 
   // ---------------- consumer warps ----------------
-  const int tsel = warp >> 2;            // which tile of the unit
-  const int mi0 = 2 * (warp & 3);        // first of two m-tiles in that tile
+  const int tsel = warp / (8 / kDecMT);              // tile of the unit
+  const int mi0 = (warp % (8 / kDecMT)) * kDecMT;    // first of the warp's m-tiles in that tile
   const int gq = lane >> 2, cq = lane & 3;
-  if (!mbar_wait(xbar, 0, p.wait_budget, abort_flag, p.err)) return;
-
-  int it = 0;
-  for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x) {
-    const int ntile = min(2, p.num_tiles - 2 * unit);
-    const bool active = tsel < ntile;
-    float acc[2][NT][4];
-    float part[2][NT][4];
+  {
+    // Per-group sums of the hidden states, for removing the operand bias.
+    const bool ok = mbar_wait(xbar, 0, p.wait_budget, abort_flag, p.err);
+    const int ng = p.d_pad / p.g;
+    if (ok) {
+      for (int e = threadIdx.x; e < ng * kDecodeMaxTokens; e += kDecWarps * 32) {
+        const int grp = e / kDecodeMaxTokens, m = e % kDecodeMaxTokens;
+        float sum = 0.f;
+        if (m < p.M) {
+          const uint32_t *row = reinterpret_cast<const uint32_t *>(xs_s + m * xrow + grp * p.g);
+          for (int k = 0; k < p.g / 2; ++k) {
+            const uint32_t v = row[k];
+            sum += bf16_lo(v);
+            sum += bf16_hi(v);
+          }
+        }
+        xsum_s[e] = -kInt4Bias * sum;
+      }
+    }
+    asm volatile("bar.sync 1, %0;\n" ::"r"(kDecWarps * 32) : "memory");  // consumer warps only
+    if (!ok) return;
+  }
+  // B-fragment bases: token 8*nt + gq (clamped to the M rows held; the extra
+  // columns are never stored), column 2*cq (+ 16 per k step, + 8 for b1).
+  const uint16_t *xb[NT];
 #pragma unroll
-    for (int a = 0; a < 2; ++a)
+  for (int nt = 0; nt < NT; ++nt) xb[nt] = xs_s + min(8 * nt + gq, p.M - 1) * xrow + 2 * cq;
+  bool t_ready = false;
+
+  int st = 0;     // ring slot
+  uint32_t ph = 0;  // its phase parity
+  for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x) {
+    const int ntile = min(kDecTiles, p.num_tiles - kDecTiles * unit);
+    const bool active = tsel < ntile;
+    float acc[kDecMT][NT][4];
+    float part[kDecMT][NT][4];  // one group's sums; each group's first MMA starts from zero
+#pragma unroll
+    for (int a = 0; a < kDecMT; ++a)
 #pragma unroll
       for (int b = 0; b < NT; ++b)
 #pragma unroll
         for (int c = 0; c < 4; ++c) acc[a][b][c] = part[a][b][c] = 0.f;
 
-    // Residual: INT4 codes, promoted per group.
-    for (int s = 0; s < res_stages; ++s, ++it) {
-      const int st = it % stages;
-      if (!mbar_wait(&full[st], (it / stages) & 1, p.wait_budget, abort_flag, p.err)) return;
-      const uint8_t *buf = stage_base + (size_t)st * kDecStageBytes;
-      const int kc0 = 2 * s;
-      const int nkc = min(2, KC - kc0);
-      const int g0 = (kc0 * kChunkK) / p.g;
+    // Residual: INT4 codes, promoted per group.  Each warp copies its share of
+    // a stage (codes and group scales) to registers and releases the slot at
+    // once, so the producer can refill it while the warp computes.
+    constexpr int NGS = GS <= SS ? SS / GS : 1;  // groups whose scales a stage carries
+    for (int s = 0; s < res_stages; ++s) {
+      if (!mbar_wait(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
+      uint4 w[SC][kDecMT];
+      float s_lo[NGS][kDecMT], s_hi[NGS][kDecMT];
       if (active) {
-        const uint16_t *sc = reinterpret_cast<const uint16_t *>(buf + kDecStageCodeBytes + tsel * 4 * kTileRows * 2);
-        for (int c = 0; c < nkc; ++c) {
-          uint4 w[2];
+        const uint8_t *buf = smem + (size_t)st * Geom::kBytes;
+        const uint8_t *cb = buf + tsel * SC * kChunkBytes + mi0 * 512 + lane * 16;
+        const uint16_t *sc = reinterpret_cast<const uint16_t *>(buf + Geom::kCodeBytes + tsel * Geom::kScaleBytesPerTile) +
+                             mi0 * 16 + gq;
 #pragma unroll
-          for (int mt = 0; mt < 2; ++mt)
-            w[mt] = *reinterpret_cast<const uint4 *>(buf + ((tsel * 2 + c) * 8 + mi0 + mt) * 512 + lane * 16);
+        for (int c = 0; c < SC; ++c)
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const int s16 = (kc0 + c) * 4 + j;
-            uint32_t b[NT][2];
+          for (int mt = 0; mt < kDecMT; ++mt) w[c][mt] = *reinterpret_cast<const uint4 *>(cb + c * kChunkBytes + mt * 512);
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-              const uint2 bb = *reinterpret_cast<const uint2 *>(
-                  xs_s + (((size_t)nt * (p.d / 32) + (s16 >> 1)) * 32 + lane) * 4 + (s16 & 1) * 2);
-              b[nt][0] = bb.x;
-              b[nt][1] = bb.y;
-            }
+        for (int gi = 0; gi < NGS; ++gi)
 #pragma unroll
-            for (int mt = 0; mt < 2; ++mt) {
-              const uint32_t word = j == 0 ? w[mt].x : j == 1 ? w[mt].y : j == 2 ? w[mt].z : w[mt].w;
-              uint32_t a[4];
-              unpack_int4x8(word, a);
-#pragma unroll
-              for (int nt = 0; nt < NT; ++nt) mma_bf16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
-            }
-            if (((s16 + 1) & ((1 << p.g_shift) - 1)) == 0) {
-              const int grp = (s16 >> p.g_shift) - g0;
-#pragma unroll
-              for (int mt = 0; mt < 2; ++mt) {
-                const int r = (mi0 + mt) * 16 + gq;
-                const float s_lo = fp16_bits_to_f32(sc[grp * kTileRows + r]);
-                const float s_hi = fp16_bits_to_f32(sc[grp * kTileRows + r + 8]);
-#pragma unroll
-                for (int nt = 0; nt < NT; ++nt) {
-                  acc[mt][nt][0] = fmaf(s_lo, part[mt][nt][0], acc[mt][nt][0]);
-                  acc[mt][nt][1] = fmaf(s_lo, part[mt][nt][1], acc[mt][nt][1]);
-                  acc[mt][nt][2] = fmaf(s_hi, part[mt][nt][2], acc[mt][nt][2]);
-                  acc[mt][nt][3] = fmaf(s_hi, part[mt][nt][3], acc[mt][nt][3]);
-#pragma unroll
-                  for (int c2 = 0; c2 < 4; ++c2) part[mt][nt][c2] = 0.f;
-                }
-              }
-            }
+          for (int mt = 0; mt < kDecMT; ++mt) {
+            s_lo[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16]);
+            s_hi[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16 + 8]);
           }
-        }
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty[st]);
-    }
-
-    // Rank-r branches as extra k steps (core: factor 1; correction: row scale of A_w).
-    for (int s = 0; s < lr_stages; ++s, ++it) {
-      const int st = it % stages;
-      if (!mbar_wait(&full[st], (it / stages) & 1, p.wait_budget, abort_flag, p.err)) return;
-      const uint8_t *buf = stage_base + (size_t)st * kDecStageBytes;
-      const int ls0 = s * kDecLrStepsPerStage;
-      const int nl = min(kDecLrStepsPerStage, p.nls - ls0);
-      if (active) {
-        for (int l = 0; l < nl; ++l) {
-          const int ls = ls0 + l;
-          uint32_t bh[NT][2], bl[NT][2];
+      if (++st == stages) st = 0, ph ^= 1;
+      if (!active) continue;
+      const int kbase = s * SS * 16;
+#pragma unroll
+      for (int c = 0; c < SC; ++c) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int ks = c * 4 + j;  // k step within the stage
+          uint32_t b[NT][2];
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
-            const uint2 h2 = *reinterpret_cast<const uint2 *>(ts_s + ((((size_t)ls * 2 + 0) * 2 + nt) * 32 + lane) * 2);
-            const uint2 l2 = *reinterpret_cast<const uint2 *>(ts_s + ((((size_t)ls * 2 + 1) * 2 + nt) * 32 + lane) * 2);
-            bh[nt][0] = h2.x;
-            bh[nt][1] = h2.y;
-            bl[nt][0] = l2.x;
-            bl[nt][1] = l2.y;
+            const uint16_t *q = xb[nt] + kbase + ks * 16;
+            b[nt][0] = *reinterpret_cast<const uint32_t *>(q);
+            b[nt][1] = *reinterpret_cast<const uint32_t *>(q + 8);
           }
 #pragma unroll
-          for (int mt = 0; mt < 2; ++mt) {
-            const uint2 w2 = *reinterpret_cast<const uint2 *>(
-                buf + (((size_t)tsel * kDecLrStepsPerStage + l) * 8 + mi0 + mt) * 256 + lane * 8);
+          for (int mt = 0; mt < kDecMT; ++mt) {
+            const uint32_t word = j == 0 ? w[c][mt].x : j == 1 ? w[c][mt].y : j == 2 ? w[c][mt].z : w[c][mt].w;
             uint32_t a[4];
-            unpack_int8x8(w2.x, w2.y, a);
+            unpack_int4x8_biased(word, a);
+            // First k step of a group: compile-time when groups fit in a stage.
+            const bool first = GS <= SS ? (ks % GS == 0) : (ks == 0 && (s % (GS / SS)) == 0);
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
-              mma_bf16_16816(part[mt][nt], a, bh[nt][0], bh[nt][1]);
-              mma_bf16_16816(part[mt][nt], a, bl[nt][0], bl[nt][1]);
+              if (first)
+                mma_bf16_16816_zero(part[mt][nt], a, b[nt][0], b[nt][1]);
+              else
+                mma_bf16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
             }
           }
-          if (ls + 1 == p.nls_core || ls + 1 == p.nls) {
-            const bool corr = ls + 1 == p.nls && p.nls > p.nls_core;
-            const uint16_t *sa = reinterpret_cast<const uint16_t *>(buf + kDecStageCodeBytes + tsel * kTileRows * 2);
+          // Group boundary: compile-time inside a stage when GS <= SS; every
+          // GS/SS stages otherwise.
+          const bool boundary = GS <= SS ? ((ks + 1) % GS == 0) : (ks == SS - 1 && ((s + 1) % (GS / SS)) == 0);
+          if (boundary) {
+            const int gi = GS <= SS ? ks / GS : 0;                               // group within the stage
+            const int ggl = GS <= SS ? s * (SS / GS) + ks / GS : s / (GS / SS);  // group index along d
+            float2 nb[NT];
 #pragma unroll
-            for (int mt = 0; mt < 2; ++mt) {
-              const int r = (mi0 + mt) * 16 + gq;
-              const float f_lo = corr ? fp16_bits_to_f32(sa[r]) : 1.f;
-              const float f_hi = corr ? fp16_bits_to_f32(sa[r + 8]) : 1.f;
+            for (int nt = 0; nt < NT; ++nt)
+              nb[nt] = *reinterpret_cast<const float2 *>(xsum_s + ggl * kDecodeMaxTokens + 8 * nt + 2 * cq);
 #pragma unroll
-              for (int nt = 0; nt < NT; ++nt) {
-                acc[mt][nt][0] = fmaf(f_lo, part[mt][nt][0], acc[mt][nt][0]);
-                acc[mt][nt][1] = fmaf(f_lo, part[mt][nt][1], acc[mt][nt][1]);
-                acc[mt][nt][2] = fmaf(f_hi, part[mt][nt][2], acc[mt][nt][2]);
-                acc[mt][nt][3] = fmaf(f_hi, part[mt][nt][3], acc[mt][nt][3]);
-#pragma unroll
-                for (int c2 = 0; c2 < 4; ++c2) part[mt][nt][c2] = 0.f;
-              }
-            }
+            for (int mt = 0; mt < kDecMT; ++mt) promote_res<NT>(acc[mt], part[mt], s_lo[gi][mt], s_hi[gi][mt], nb);
           }
+        }
+      }
+    }
+
+    // Rank-r branches as extra k steps (core: factor 1; correction: row scale
+    // of A_w), with the same copy-then-release of each stage.
+#pragma unroll
+    for (int a = 0; a < kDecMT; ++a)
+#pragma unroll
+      for (int b = 0; b < NT; ++b)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) part[a][b][c] = 0.f;
+    for (int s = 0; s < lr_stages; ++s) {
+      if (!t_ready) {
+        if (!mbar_wait(tbar, 0, p.wait_budget, abort_flag, p.err)) return;
+        t_ready = true;
+      }
+      if (!mbar_wait(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
+      const int ls0 = s * Geom::kLrSteps;
+      const int nl = min(Geom::kLrSteps, p.nls - ls0);
+      const bool last_stage = s == lr_stages - 1;
+      uint2 lw[Geom::kLrSteps][kDecMT];
+      float a_lo[kDecMT], a_hi[kDecMT];
+      if (active) {
+        const uint8_t *buf = smem + (size_t)st * Geom::kBytes;
+#pragma unroll
+        for (int l = 0; l < Geom::kLrSteps; ++l)
+#pragma unroll
+          for (int mt = 0; mt < kDecMT; ++mt)
+            if (l < nl)
+              lw[l][mt] = *reinterpret_cast<const uint2 *>(
+                  buf + ((size_t)(tsel * Geom::kLrSteps + l) * 8 + mi0 + mt) * 256 + lane * 8);
+        const uint16_t *sa = reinterpret_cast<const uint16_t *>(buf + Geom::kCodeBytes + tsel * Geom::kScaleBytesPerTile);
+#pragma unroll
+        for (int mt = 0; mt < kDecMT; ++mt) {
+          const int r = (mi0 + mt) * 16 + gq;
+          a_lo[mt] = last_stage ? fp16_bits_to_f32(sa[r]) : 0.f;
+          a_hi[mt] = last_stage ? fp16_bits_to_f32(sa[r + 8]) : 0.f;
         }
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty[st]);
+      if (++st == stages) st = 0, ph ^= 1;
+      if (!active) continue;
+#pragma unroll
+      for (int l = 0; l < Geom::kLrSteps; ++l) {
+        if (l >= nl) break;
+        const int ls = ls0 + l;
+        uint32_t bh[NT][2], bl[NT][2];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          const uint2 h2 = *reinterpret_cast<const uint2 *>(ts_s + ((((size_t)ls * 2 + 0) * 2 + nt) * 32 + lane) * 2);
+          const uint2 l2 = *reinterpret_cast<const uint2 *>(ts_s + ((((size_t)ls * 2 + 1) * 2 + nt) * 32 + lane) * 2);
+          bh[nt][0] = h2.x;
+          bh[nt][1] = h2.y;
+          bl[nt][0] = l2.x;
+          bl[nt][1] = l2.y;
+        }
+#pragma unroll
+        for (int mt = 0; mt < kDecMT; ++mt) {
+          uint32_t a[4];
+          unpack_int8x8(lw[l][mt].x, lw[l][mt].y, a);
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            mma_bf16_16816(part[mt][nt], a, bh[nt][0], bh[nt][1]);
+            mma_bf16_16816(part[mt][nt], a, bl[nt][0], bl[nt][1]);
+          }
+        }
+        if (ls + 1 == p.nls_core || ls + 1 == p.nls) {
+          const bool corr = ls + 1 == p.nls && p.nls > p.nls_core;  // the correction ends with the last stage
+#pragma unroll
+          for (int mt = 0; mt < kDecMT; ++mt) {
+            promote<NT>(acc[mt], part[mt], corr ? a_lo[mt] : 1.f, corr ? a_hi[mt] : 1.f);
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+              for (int c = 0; c < 4; ++c) part[mt][nt][c] = 0.f;
+          }
+        }
+      }
     }
 
     // Epilogue.  acc[mt][nt][i]: row 16*(mi0+mt) + gq + 8*(i/2), token 8*nt + 2*cq + i%2.
-    const int64_t row_base = (2 * (int64_t)unit + tsel) * kTileRows;
+    const int64_t row_base = ((int64_t)kDecTiles * unit + tsel) * kTileRows;
     if (p.out) {
       if (active) {
 #pragma unroll
-        for (int mt = 0; mt < 2; ++mt)
+        for (int mt = 0; mt < kDecMT; ++mt)
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
@@ -291,28 +431,29 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
             }
       }
     } else {
-      // Cross-entropy partials: per (warp, token) running max and sum of exp.
+      // Cross-entropy partials: per (unit, warp, token) running max and sum of exp.
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
         for (int tl = 0; tl < 2; ++tl) {
           const int tok = nt * 8 + 2 * cq + tl;
           const int tgt = tok < p.M ? p.targets[p.m0 + tok] : -1;
-          float vals[4];
+          float vals[2 * kDecMT];
           float mx = -INFINITY;
 #pragma unroll
-          for (int mt = 0; mt < 2; ++mt)
+          for (int mt = 0; mt < kDecMT; ++mt)
 #pragma unroll
             for (int ih = 0; ih < 2; ++ih) {
               const int64_t row = row_base + (mi0 + mt) * 16 + gq + 8 * ih;
-              const float v = (active && row < p.V) ? acc[mt][nt][ih * 2 + tl] : -INFINITY;
+              const bool ok = active && row < p.V;
+              const float v = ok ? acc[mt][nt][ih * 2 + tl] : -INFINITY;
               vals[mt * 2 + ih] = v;
               mx = fmaxf(mx, v);
-              if (active && row < p.V && row == tgt) p.ce_tlogit[p.m0 + tok] = v;
+              if (ok && row == tgt) p.ce_tlogit[p.m0 + tok] = v;
             }
           float sum = 0.f;
 #pragma unroll
-          for (int q = 0; q < 4; ++q) sum += (vals[q] == -INFINITY) ? 0.f : __expf(vals[q] - mx);
+          for (int q = 0; q < 2 * kDecMT; ++q) sum += (vals[q] == -INFINITY) ? 0.f : __expf(vals[q] - mx);
           LsePair lp{mx, sum};
 #pragma unroll
           for (int off = 4; off < 32; off <<= 1) {
@@ -320,34 +461,59 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
             lp = lse_merge(lp, o);
           }
           if (gq == 0 && tok < p.M)
-            p.ce_part[((int64_t)unit * kDecConsumerWarps + warp) * p.M_total + p.m0 + tok] = make_float2(lp.m, lp.s);
+            p.ce_part[((int64_t)unit * kDecWarps + warp) * p.M_total + p.m0 + tok] = make_float2(lp.m, lp.s);
         }
     }
   }
 }
 
-int decode_num_units(const archead_pack *p) { return (p->num_tiles + 1) / 2; }
+int decode_num_units(const archead_pack *p) { return (p->num_tiles + kDecTiles - 1) / kDecTiles; }
 
-int decode_parts_per_unit() { return kDecConsumerWarps; }
+int decode_parts_per_unit() { return kDecWarps; }
 
-bool decode_supported(int d, int nls) { return decode_plan(d, nls, 2).stages >= 2; }
+bool decode_supported(int d_pad, int nls, int g) { return decode_plan(d_pad, nls, g, kDecodeMaxTokens).stages >= 2; }
 
-cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s) {
-  const DecodeSmemPlan pl = decode_plan(dp.d, dp.nls, dp.NT);
-  if (pl.stages < 2) return cudaErrorInvalidValue;
-  cudaError_t e;
-  if (dp.NT == 1) {
-    e = cudaFuncSetAttribute(decode_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.total);
+template <int NT, int SC, int GS>
+static cudaError_t launch_t(const DecodeParams &dp, int grid, cudaStream_t s, const DecodePlan &pl, bool pdl) {
+  auto kern = decode_kernel<NT, SC, GS>;
+  static int smem_set = 0;  // largest dynamic shared memory opted in so far for this instance
+  if ((int)pl.total > smem_set) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.total);
     if (e != cudaSuccess) return e;
-    decode_kernel<1><<<grid, kDecThreads, pl.total, s>>>(dp, pl.stages, (int)pl.xs_off, (int)pl.ts_off,
-                                                         (int)pl.bar_off);
-  } else {
-    e = cudaFuncSetAttribute(decode_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.total);
-    if (e != cudaSuccess) return e;
-    decode_kernel<2><<<grid, kDecThreads, pl.total, s>>>(dp, pl.stages, (int)pl.xs_off, (int)pl.ts_off,
-                                                         (int)pl.bar_off);
+    smem_set = (int)pl.total;
   }
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kDecThreads);
+  cfg.dynamicSmemBytes = pl.total;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, dp, pl.stages, (int)pl.xs_off, (int)pl.ts_off, (int)pl.xsum_off,
+                            (int)pl.bar_off);
+}
+
+template <int NT, int SC>
+static cudaError_t launch_g(const DecodeParams &dp, int grid, cudaStream_t s, const DecodePlan &pl, bool pdl) {
+  switch (dp.g) {
+    case 32: return launch_t<NT, SC, 2>(dp, grid, s, pl, pdl);
+    case 64: return launch_t<NT, SC, 4>(dp, grid, s, pl, pdl);
+    case 128: return launch_t<NT, SC, 8>(dp, grid, s, pl, pdl);
+    case 256: return launch_t<NT, SC, 16>(dp, grid, s, pl, pdl);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool pdl) {
+  const DecodePlan pl = decode_plan(dp.d_pad, dp.nls, dp.g, dp.M);
+  if (pl.stages < 2) return cudaErrorInvalidValue;
+  static_assert(stage_chunks(1) >= 1 && stage_chunks(2) >= 1, "stage width");
+  if ((dp.NT == 1) != (dp.M <= 8) || pl.sc != stage_chunks(dp.NT)) return cudaErrorInvalidValue;
+  if (dp.NT == 1) return launch_g<1, stage_chunks(1)>(dp, grid, s, pl, pdl);
+  return launch_g<2, stage_chunks(2)>(dp, grid, s, pl, pdl);
 }
 
 }  // namespace archead

@@ -18,23 +18,42 @@ constexpr int kErrTargetRange = 2;
 //
 // Residual codes are stored offset-binary (code + 8, 0..15) in the tiled
 // layout.  Nibbles i and i+4 of a 32-bit word form bf16 pair i: OR-ing the
-// nibble into the mantissa of bf16 128.0 gives 128 + (code + 8) exactly, and
-// subtracting 136.0 (exact in bf16) leaves the code.  The two halves of each
-// output register are the (lower, higher) k of one operand pair.
+// nibble into the mantissa of bf16 128.0 gives 128 + (code + 8) exactly.  The
+// two halves of each output register are the (lower, higher) k of one pair.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t bf16x2_sub(uint32_t a, uint32_t b) {
   __nv_bfloat162 r = __hsub2(*reinterpret_cast<__nv_bfloat162 *>(&a), *reinterpret_cast<__nv_bfloat162 *>(&b));
   return *reinterpret_cast<uint32_t *>(&r);
 }
 
+// (a & b) | c in one LOP3.  Written out because the compiler splits the
+// expression into two logic operations when b and c are both immediates.
+__device__ __forceinline__ uint32_t lop3_and_or(uint32_t a, uint32_t b, uint32_t c) {
+  uint32_t d;
+  asm("lop3.b32 %0, %1, %2, %3, 0xEA;\n" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
+
+// Biased operands: each half is 136 + code (128..143, exact in bf16).  The
+// decode kernel multiplies these directly and removes 136 * sum(x) per group
+// in fp32 at promotion time.
+__device__ __forceinline__ void unpack_int4x8_biased(uint32_t w, uint32_t (&a)[4]) {
+  const uint32_t kMask = 0x000F000Fu;
+  const uint32_t kMagic = 0x43004300u;  // bf16 128.0 | 128.0
+  a[0] = lop3_and_or(w, kMask, kMagic);
+  a[1] = lop3_and_or(w >> 4, kMask, kMagic);
+  a[2] = lop3_and_or(w >> 8, kMask, kMagic);
+  a[3] = lop3_and_or(w >> 12, kMask, kMagic);
+}
+
+constexpr float kInt4Bias = 136.0f;
+
+// Exact codes: the biased operands minus 136.0 (exact in bf16).
 __device__ __forceinline__ void unpack_int4x8(uint32_t w, uint32_t (&a)[4]) {
-  constexpr uint32_t kMask = 0x000F000Fu;
-  constexpr uint32_t kMagic = 0x43004300u;  // bf16 128.0 | 128.0
-  constexpr uint32_t kBias = 0x43084308u;   // bf16 136.0 | 136.0
-  a[0] = bf16x2_sub((w & kMask) | kMagic, kBias);
-  a[1] = bf16x2_sub(((w >> 4) & kMask) | kMagic, kBias);
-  a[2] = bf16x2_sub(((w >> 8) & kMask) | kMagic, kBias);
-  a[3] = bf16x2_sub(((w >> 12) & kMask) | kMagic, kBias);
+  constexpr uint32_t kBias = 0x43084308u;  // bf16 136.0 | 136.0
+  unpack_int4x8_biased(w, a);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) a[i] = bf16x2_sub(a[i], kBias);
 }
 
 // INT8 codes are stored offset-binary (code + 128).  Placing byte u in the
@@ -75,6 +94,15 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a
       "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Same with a zero accumulator input (the first k step of a group).
+__device__ __forceinline__ void mma_bf16_16816_zero(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%10,%10,%10};\n"
+      : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(0.f));
 }
 
 // ---------------------------------------------------------------------------

@@ -3,15 +3,17 @@
 // Device layouts (all built by archead_pack_create from the canonical layout):
 //
 //  Residual codes, "fragment-native" tiling.  The vocabulary is cut into
-//  tiles of 128 rows (V padded with zero rows), d into chunks of 64.  Chunk
+//  tiles of 128 rows (V padded with zero rows), d (padded with zero codes to
+//  D_PAD, a multiple of 128) into chunks of 64.  Chunk
 //  (vt, kc) is 4 KB: [mi 0..7][lane 0..31][word j 0..3] of 32-bit words.
 //  Word j of lane (gq = lane/4, cq = lane%4) in m-tile mi holds the 8 codes an
 //  m16n8k16 A-fragment needs for k16-step 4*kc + j: nibble p (pair i = p%4,
 //  half h = p/4) is row 16*mi + gq + 8*(i%2), column 16*(4*kc+j) + 2*cq +
 //  8*(i/2) + h.  Codes are stored offset-binary (code + 8).
-//    byte offset = ((((vt*KC + kc)*8 + mi)*32 + lane)*4 + j)*4,   KC = d/64
+//    byte offset = ((((vt*KC + kc)*8 + mi)*32 + lane)*4 + j)*4,   KC = D_PAD/64
 //
-//  Residual scales: [vt][G][128] fp16 bits (row within tile fastest).
+//  Residual scales: [vt][G_PAD][128] fp16 bits (row within tile fastest),
+//  G_PAD = D_PAD/g; scales of padding groups and rows are zero.
 //
 //  Low-rank codes: the extended rank axis kk in [0, LR) with LR = RCP + RRP,
 //  RCP = r_c rounded up to 32, RRP = r_r rounded up to 32: kk < RCP is
@@ -47,10 +49,10 @@ struct DecodeParams {
   const uint16_t *scales;
   const uint8_t *lr_codes;
   const uint16_t *s_a;
-  const uint32_t *xs;   // x fragments for this token chunk
+  const uint16_t *x;    // hidden states [M_total][d] bf16 (this chunk starts at row m0)
   const uint32_t *ts;   // t hi/lo fragments for this token chunk
   int64_t V;
-  int num_tiles, d, G, g, g_shift, nls, nls_core;  // g_shift = log2(g / 16)
+  int num_tiles, d, d_pad, G_pad, g, nls, nls_core;
   int M;                // tokens in this chunk (1..16)
   int m0;               // index of the chunk's first token
   int NT;               // n-tiles of 8 tokens (1 or 2)
@@ -72,11 +74,10 @@ struct PrepassParams {
   const uint16_t *s_b;     // [G][r_r]
   const uint16_t *s_u, *s_v;
   int M, d, g, rc, rr, rcp, rrp, lr;
-  float *partial;          // [d/256][M][LR]
-  // outputs of finalize
+  float *partial;          // per-split partial sums (workspace)
+  int *counters;           // one per (columns, tokens) block pair, zero between calls
   uint32_t *ts;            // decode t fragments, per 16-token chunk
   uint16_t *T;             // prefill extended-K operand [M][2*LR] bf16 (may be NULL)
-  uint32_t *xs;            // decode x fragments, per 16-token chunk (may be NULL)
 };
 
 struct KernelTimer {
@@ -93,6 +94,7 @@ struct archead_pack {
   int sm_count = 0;
   int64_t V = 0, V_pad = 0;
   int d = 0, rc = 0, rr = 0, g = 0, G = 0, rcp = 0, rrp = 0, lr = 0, nls = 0, nls_core = 0;
+  int d_pad = 0, G_pad = 0;  // d rounded up to 128, and its group count
   int num_tiles = 0;
   // device buffers owned by the pack
   uint8_t *codes = nullptr;
@@ -103,9 +105,11 @@ struct archead_pack {
   uint16_t *s_u = nullptr, *s_v = nullptr, *s_b = nullptr;
   int *err = nullptr;
   int64_t owned_bytes = 0;
-  // workspace (grown on demand)
+  // workspace (grown on demand) and the pre-pass block counters (kept zero)
   void *ws = nullptr;
   size_t ws_bytes = 0;
+  int *counters = nullptr;
+  int counters_len = 0;
   // host staging for archead_forward_host
   void *xh_dev = nullptr, *yh_dev = nullptr;
   size_t xh_bytes = 0, yh_bytes = 0;
@@ -123,10 +127,14 @@ cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, cons
 cudaError_t launch_debug_dequant(const archead_pack *p, int comp, int64_t row0, int64_t nrows, float *out,
                                  cudaStream_t s);
 cudaError_t launch_prepass(const PrepassParams &pp, cudaStream_t s, archead_pack *p);
-cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s);
+int prepass_pairs(int M, int lr);
+size_t prepass_smem(int M);  // dynamic shared memory of one pre-pass block
+size_t prepass_partial_bytes(int M, int lr, int d);
+// pdl: launch as a programmatic dependent of the immediately preceding pre-pass grid.
+cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool pdl);
 int decode_num_units(const archead_pack *p);
 int decode_parts_per_unit();
-bool decode_supported(int d, int nls);
+bool decode_supported(int d_pad, int nls, int g);
 cudaError_t launch_ce_finalize(const float2 *part, int num_parts, const float *tlogit, const int32_t *targets,
                                int64_t V, int M, float *ce, int *err, cudaStream_t s);
 cudaError_t launch_wait_timeout_probe(int *err, int64_t budget, cudaStream_t s);

@@ -8,15 +8,17 @@ namespace archead {
 
 // One block per (vocabulary tile, 64-wide chunk of d): stage the canonical
 // 128 x 32 bytes in shared memory, then emit the 1024 fragment words.
-__global__ void build_res_codes_kernel(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst, int64_t V, int d) {
+__global__ void build_res_codes_kernel(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst, int64_t V, int d,
+                                       int d_pad) {
   __shared__ uint8_t tile[kTileRows][kChunkK / 2];
-  const int KC = d / kChunkK;
+  const int KC = d_pad / kChunkK;
   const int vt = blockIdx.x / KC;
   const int kc = blockIdx.x % KC;
   for (int i = threadIdx.x; i < kTileRows * (kChunkK / 2); i += blockDim.x) {
     int r = i / (kChunkK / 2), b = i % (kChunkK / 2);
     int64_t row = (int64_t)vt * kTileRows + r;
-    tile[r][b] = row < V ? src[row * (d / 2) + (int64_t)kc * (kChunkK / 2) + b] : (uint8_t)0x88;  // code 0
+    // Padding rows and padding columns (k >= d; d is a multiple of 64) hold code 0.
+    tile[r][b] = (row < V && kc * kChunkK < d) ? src[row * (d / 2) + (int64_t)kc * (kChunkK / 2) + b] : (uint8_t)0;
   }
   __syncthreads();
   uint32_t *out = reinterpret_cast<uint32_t *>(dst) + ((int64_t)vt * KC + kc) * 1024;
@@ -37,14 +39,14 @@ __global__ void build_res_codes_kernel(const uint8_t *__restrict__ src, uint8_t 
 }
 
 __global__ void build_res_scales_kernel(const uint16_t *__restrict__ src, uint16_t *__restrict__ dst, int64_t V,
-                                        int64_t V_pad, int G) {
-  const int64_t total = V_pad * G;
+                                        int64_t V_pad, int G, int G_pad) {
+  const int64_t total = V_pad * G_pad;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
     const int64_t r = i % kTileRows;
-    const int64_t grp = (i / kTileRows) % G;
-    const int64_t vt = i / ((int64_t)kTileRows * G);
+    const int64_t grp = (i / kTileRows) % G_pad;
+    const int64_t vt = i / ((int64_t)kTileRows * G_pad);
     const int64_t row = vt * kTileRows + r;
-    dst[i] = row < V ? src[row * G + grp] : (uint16_t)0;
+    dst[i] = (row < V && grp < G) ? src[row * G + grp] : (uint16_t)0;
   }
 }
 
@@ -81,9 +83,9 @@ __global__ void build_row_scales_kernel(const uint16_t *__restrict__ src, uint16
 cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, const uint16_t *res_scales,
                                  const int8_t *core_u, const int8_t *corr_a, const uint16_t *corr_a_scale,
                                  cudaStream_t s) {
-  const int KC = p->d / kChunkK;
-  build_res_codes_kernel<<<p->num_tiles * KC, 256, 0, s>>>(res_codes, p->codes, p->V, p->d);
-  build_res_scales_kernel<<<1024, 256, 0, s>>>(res_scales, p->scales, p->V, p->V_pad, p->G);
+  const int KC = p->d_pad / kChunkK;
+  build_res_codes_kernel<<<p->num_tiles * KC, 256, 0, s>>>(res_codes, p->codes, p->V, p->d, p->d_pad);
+  build_res_scales_kernel<<<1024, 256, 0, s>>>(res_scales, p->scales, p->V, p->V_pad, p->G, p->G_pad);
   if (p->nls > 0)
     build_lr_codes_kernel<<<p->num_tiles * p->nls, 256, 0, s>>>(core_u, corr_a, p->lr_codes, p->V, p->rc, p->rr,
                                                                  p->rcp, p->nls);
@@ -100,7 +102,7 @@ struct DequantArgs {
   const uint8_t *lr_codes;
   const uint16_t *s_a, *s_u, *s_v, *s_b;
   const int8_t *q_v, *q_b;
-  int d, G, g, rc, rr, rcp, nls;
+  int d, d_pad, G_pad, g, rc, rr, rcp, nls;
 };
 
 // Position of (row-in-tile, column-in-16-step) inside a fragment: returns the
@@ -133,13 +135,13 @@ __global__ void debug_dequant_kernel(DequantArgs a, int comp, int64_t row0, int6
         const int kc = col / kChunkK, kl = col % kChunkK;
         const int j = kl >> 4;
         const int lane = frag_pos(r, kl & 15, i, h);
-        const int KC = a.d / kChunkK;
+        const int KC = a.d_pad / kChunkK;
         const uint32_t w = reinterpret_cast<const uint32_t *>(
             a.codes)[((((int64_t)vt * KC + kc) * 8 + mi) * 32 + lane) * 4 + j];
         uint32_t q[4];
-        unpack_int4x8(w, q);
+        unpack_int4x8_biased(w, q);  // the decode kernel's operands: 136 + code
         const int grp = col / a.g;
-        v = pair_half(q[i], h) * fp16_bits_to_f32(a.scales[((int64_t)vt * a.G + grp) * kTileRows + r]);
+        v = (pair_half(q[i], h) - kInt4Bias) * fp16_bits_to_f32(a.scales[((int64_t)vt * a.G_pad + grp) * kTileRows + r]);
       } else {
         const int kk = comp == 1 ? col : a.rcp + col;
         const int ls = kk >> 4;
@@ -163,7 +165,7 @@ __global__ void debug_dequant_kernel(DequantArgs a, int comp, int64_t row0, int6
 cudaError_t launch_debug_dequant(const archead_pack *p, int comp, int64_t row0, int64_t nrows, float *out,
                                  cudaStream_t s) {
   DequantArgs a{p->codes, p->scales, p->lr_codes, p->s_a, p->s_u, p->s_v, p->s_b, p->q_v, p->q_b,
-                p->d,     p->G,      p->g,        p->rc,  p->rr,  p->rcp, p->nls};
+                p->d,     p->d_pad,  p->G_pad,    p->g,   p->rc,  p->rr,  p->rcp, p->nls};
   const int cols = comp == 0 ? p->d : ((comp == 1 || comp == 2) ? p->rc : p->rr);
   const int64_t total = nrows * cols;
   if (total == 0) return cudaSuccess;
