@@ -217,14 +217,52 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   return ARCHEAD_OK;
 }
 
+// Prefill path: rank-r pre-pass into the extended operand T, then the
+// tensor-core kernel.  out == nullptr selects CE mode.
+archead_status run_prefill(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
+                           const int32_t *targets, float *ce, cudaStream_t s) {
+  const bool ce_mode = out == nullptr;
+  Carve c;
+  const size_t partial_off = c.take(prepass_partial_bytes((int)M, p->lr, p->d));
+  const size_t t_off = c.take((size_t)M * std::max(2 * p->lr, 64) * 2);
+  size_t ce_part_off = 0, tlogit_off = 0;
+  if (ce_mode) {
+    ce_part_off = c.take((size_t)p->num_tiles * prefill_parts_per_vt() * M * sizeof(float2));
+    tlogit_off = c.take((size_t)M * sizeof(float));
+  }
+  AH_CUDA(ensure_workspace(p, c.off, s));
+  AH_CUDA(ensure_counters(p, prepass_pairs((int)M, p->lr), s));
+  PrepassParams pp = prepass_params(p, x, M);
+  pp.partial = at<float>(p->ws, partial_off);
+  pp.counters = p->counters;
+  pp.ts = nullptr;
+  pp.T = at<uint16_t>(p->ws, t_off);
+  AH_CUDA(launch_prepass(pp, s, p));
+  float2 *ce_part = ce_mode ? at<float2>(p->ws, ce_part_off) : nullptr;
+  float *tlogit = ce_mode ? at<float>(p->ws, tlogit_off) : nullptr;
+  cudaEvent_t ev = nullptr;
+  timer_begin(p, "prefill", s, &ev);
+  cudaError_t e = launch_prefill(p, x, (int)M, pp.T, out, out_fp32, targets, ce_part, tlogit, s);
+  timer_end(p, "prefill", s, ev);
+  if (e != cudaSuccess) return cuda_status(e);
+  if (ce_mode) {
+    timer_begin(p, "ce_finalize", s, &ev);
+    e = launch_ce_finalize(ce_part, p->num_tiles * prefill_parts_per_vt(), tlogit, targets, p->V, (int)M, ce, p->err,
+                           s);
+    timer_end(p, "ce_finalize", s, ev);
+    if (e != cudaSuccess) return cuda_status(e);
+  }
+  return ARCHEAD_OK;
+}
+
 archead_status run_forward(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
                            const int32_t *targets, float *ce, archead_path path, cudaStream_t s) {
   if (path != ARCHEAD_PATH_AUTO && path != ARCHEAD_PATH_DECODE && path != ARCHEAD_PATH_PREFILL)
     return ARCHEAD_ERR_INVALID_ARG;
   AH_CUDA(cudaSetDevice(p->device));
-  // The tensor-core prefill kernel takes M > 16 when available; the decode
-  // kernel serves every M, sixteen tokens per pass.
-  return run_decode(p, x, M, out, out_fp32, targets, ce, s);
+  const bool decode = path == ARCHEAD_PATH_DECODE || (path == ARCHEAD_PATH_AUTO && M <= kDecodeMaxTokens);
+  if (decode) return run_decode(p, x, M, out, out_fp32, targets, ce, s);
+  return run_prefill(p, x, M, out, out_fp32, targets, ce, s);
 }
 
 }  // namespace

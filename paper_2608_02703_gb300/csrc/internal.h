@@ -135,6 +135,9 @@ cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool
 int decode_num_units(const archead_pack *p);
 int decode_parts_per_unit();
 bool decode_supported(int d_pad, int nls, int g);
+cudaError_t launch_prefill(const archead_pack *pk, const void *x, int M, const uint16_t *T, void *out, int out_fp32,
+                           const int32_t *targets, float2 *ce_part, float *ce_tlogit, cudaStream_t s);
+int prefill_parts_per_vt();
 cudaError_t launch_ce_finalize(const float2 *part, int num_parts, const float *tlogit, const int32_t *targets,
                                int64_t V, int M, float *ce, int *err, cudaStream_t s);
 cudaError_t launch_wait_timeout_probe(int *err, int64_t budget, cudaStream_t s);
