@@ -203,6 +203,28 @@ ARCHEAD_API archead_status archead_set_wait_budget(archead_pack *pack, int64_t c
  */
 ARCHEAD_API archead_status archead_debug_wait_timeout(archead_pack *pack, void *stream);
 
+/*
+ * Allocation-free variant of archead_forward for M <= 16 (the decode path).
+ * The paper has no counterpart; this exists for callers that must not
+ * allocate device memory while they run the head (all memory reserved up
+ * front, a stream being captured into a CUDA graph under a pool that forbids
+ * new allocations, latency-critical loops that cannot take cudaMalloc's locks
+ * or cudaFree's device synchronisation).  archead_forward grows the pack's
+ * workspace with cudaMalloc; this call never allocates: its scratch lives in
+ * one fixed 512 KiB array compiled into the library, which every device that
+ * loads the library holds until the process exits.
+ *   x       device, bf16 [M][d];  logits device, [M][V] (bf16 or fp32), as archead_forward.
+ * The first call on a device looks up that array's device address; make that
+ * first call before any stream capture.  All calls on a device share the
+ * array: calls whose work overlaps on the GPU (other streams, other packs at
+ * the same time) race.  Returns ARCHEAD_ERR_UNSUPPORTED (see
+ * archead_last_error) when M > 16 or the head needs more than 512 KiB of
+ * scratch (pre-pass partial sums: 2 KB per 32 rank columns per 256 of d, plus
+ * 1 KB per 16 rank columns; 174 KB for d=4096, r_c+r_r=160).
+ */
+ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pack *pack, const void *x, int64_t M,
+                                                          void *logits, archead_out_dtype out_dtype, void *stream);
+
 /* Per-kernel timing with CUDA events on the launch stream (off by default). */
 typedef struct {
   const char *name;  /* static string */

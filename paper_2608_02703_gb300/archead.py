@@ -39,6 +39,7 @@ EXPORTED = (
     "archead_forward_ce_path", "archead_forward_host", "archead_pack_bytes", "archead_device_bytes",
     "archead_debug_dequant", "archead_sync_status", "archead_set_wait_budget", "archead_debug_wait_timeout",
     "archead_profile_enable", "archead_profile_read", "archead_status_string", "archead_last_error",
+    "archead_forward_decode_noalloc",
 )
 
 
@@ -47,7 +48,7 @@ class ArcheadError(RuntimeError):
         self.status = status
         msg = f"{where}: {_status_string(status)}"
         detail = _last_error()
-        if status == ERR_CUDA and detail:
+        if status in (ERR_CUDA, ERR_UNSUPPORTED) and detail:
             msg += f" ({detail})"
         super().__init__(msg)
 
@@ -93,6 +94,7 @@ def load() -> ctypes.CDLL:
         "archead_forward_ce": (i32, [vp, vp, i64, vp, vp, vp]),
         "archead_forward_ce_path": (i32, [vp, vp, i64, vp, vp, i32, vp]),
         "archead_forward_host": (i32, [vp, vp, i64, vp, i32, vp]),
+        "archead_forward_decode_noalloc": (i32, [vp, vp, i64, vp, i32, vp]),
         "archead_pack_bytes": (i64, [vp]),
         "archead_device_bytes": (i64, [vp]),
         "archead_debug_dequant": (i32, [vp, i32, i64, i64, vp, vp]),
@@ -205,6 +207,12 @@ def archead_forward_ce_path(pack: Pack, x, M: int, targets, ce, path: int, strea
 def archead_forward_host(pack: Pack, x_host, M: int, logits_host, out_dtype: int = OUT_BF16, stream=None) -> None:
     _check(load().archead_forward_host(pack.handle, _ptr(x_host), M, _ptr(logits_host), out_dtype,
                                        _stream_ptr(stream)), "archead_forward_host")
+
+
+def archead_forward_decode_noalloc(pack: Pack, x, M: int, logits, out_dtype: int = OUT_BF16, stream=None) -> None:
+    """archead_forward for M <= 16 without any device allocation (fixed 512 KiB scratch array in the library)."""
+    _check(load().archead_forward_decode_noalloc(pack.handle, _ptr(x), M, _ptr(logits), out_dtype,
+                                                 _stream_ptr(stream)), "archead_forward_decode_noalloc")
 
 
 def archead_pack_bytes(pack: Pack) -> int:

@@ -269,6 +269,8 @@ archead_status run_forward(archead_pack *p, const void *x, int64_t M, void *out,
 
 namespace archead {
 
+void set_last_error_message(const char *msg) { g_last_error = msg ? msg : ""; }
+
 void timer_begin(archead_pack *p, const char *name, cudaStream_t s, cudaEvent_t *ev0) {
   *ev0 = nullptr;
   if (!p || !p->profiling) return;

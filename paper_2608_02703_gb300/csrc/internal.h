@@ -142,6 +142,9 @@ cudaError_t launch_ce_finalize(const float2 *part, int num_parts, const float *t
                                int64_t V, int M, float *ce, int *err, cudaStream_t s);
 cudaError_t launch_wait_timeout_probe(int *err, int64_t budget, cudaStream_t s);
 
+// Message returned by archead_last_error() for this thread.
+void set_last_error_message(const char *msg);
+
 // Profiling hooks (no-ops unless profiling is enabled on the pack).
 void timer_begin(archead_pack *p, const char *name, cudaStream_t s, cudaEvent_t *ev0);
 void timer_end(archead_pack *p, const char *name, cudaStream_t s, cudaEvent_t ev0);

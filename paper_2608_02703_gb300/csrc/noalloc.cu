@@ -1,0 +1,153 @@
+// Allocation-free decode forward (archead_forward_decode_noalloc).
+//
+// Who needs it: callers that must not allocate device memory while they run
+// the head -- a serving loop that reserved all device memory up front for its
+// KV cache and weights, code that runs while a CUDA graph is being captured on
+// a stream whose pool forbids new allocations, or a latency-critical loop that
+// cannot afford cudaMalloc / cudaFree (both take allocator locks and cudaFree
+// synchronises the device).  archead_forward grows a per-pack workspace with
+// cudaMalloc the first time it sees a larger M; this entry point never does.
+//
+// It runs the same pre-pass and decode kernels as archead_forward for
+// M <= 16, but takes every scratch buffer (the pre-pass's per-split partial
+// sums, its block counters and the rank-r B fragments) from one fixed array
+// compiled into the library, g_noalloc_scratch, of kNoallocScratchBytes.
+// Every device that loads the library holds this array until the process
+// exits.  All calls on a device share it and it keeps the previous call's
+// contents; the counters that must start at zero are cleared on the stream at
+// the start of each call, everything else is fully rewritten before it is
+// read.  Two calls whose work overlaps on the GPU (different streams, or
+// different packs on the same device at the same time) race on the array.
+#include <cuda_runtime.h>
+
+#include <mutex>
+
+#include "device.cuh"
+#include "internal.h"
+
+namespace archead {
+
+constexpr size_t kNoallocScratchBytes = (size_t)512 << 10;  // 512 KiB
+constexpr size_t kNoallocCounterBytes = 4096;              // 1024 block counters
+constexpr int kNoallocMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
+
+// Device address of g_noalloc_scratch, resolved once per device with that
+// device current.  In host code the symbol is only a host-side stand-in: a
+// kernel handed &g_noalloc_scratch would fault (or silently touch host memory
+// where the device can reach it), so kernels only ever get this address.
+static void *g_scratch_dev[kNoallocMaxDevices];
+static std::mutex g_scratch_mu;
+
+static cudaError_t scratch_address(int device, void **out) {
+  if (device < 0 || device >= kNoallocMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_dev[device]) {
+    void *ptr = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+    if (e != cudaSuccess) return e;
+    g_scratch_dev[device] = ptr;
+  }
+  *out = g_scratch_dev[device];
+  return cudaSuccess;
+}
+
+}  // namespace archead
+
+using namespace archead;
+
+extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pack *pack, const void *x, int64_t M,
+                                                                     void *logits, archead_out_dtype out_dtype,
+                                                                     void *stream) {
+  if (!pack || M < 0) return ARCHEAD_ERR_INVALID_ARG;
+  if (M == 0) return ARCHEAD_OK;
+  if (!x || !logits || (reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(logits) & 15))
+    return ARCHEAD_ERR_INVALID_ARG;
+  if (out_dtype != ARCHEAD_OUT_BF16 && out_dtype != ARCHEAD_OUT_FP32) return ARCHEAD_ERR_INVALID_ARG;
+  if (M > kDecodeMaxTokens) {
+    set_last_error_message("archead_forward_decode_noalloc: M must be at most 16");
+    return ARCHEAD_ERR_UNSUPPORTED;
+  }
+  if (!decode_supported(pack->d_pad, pack->nls, pack->g)) {
+    set_last_error_message("archead_forward_decode_noalloc: the decode kernel does not support this head shape");
+    return ARCHEAD_ERR_UNSUPPORTED;
+  }
+  // Scratch: [block counters | pre-pass partial sums | rank-r fragments of one 16-token chunk].
+  const int pairs = prepass_pairs((int)M, pack->lr);
+  const size_t partial_bytes = (prepass_partial_bytes((int)M, pack->lr, pack->d) + 255) / 256 * 256;
+  const size_t ts_bytes = (size_t)(pack->nls > 0 ? pack->nls : 1) * 1024;
+  const size_t need = kNoallocCounterBytes + partial_bytes + ts_bytes;
+  if (need > kNoallocScratchBytes || (size_t)pairs * sizeof(int) > kNoallocCounterBytes) {
+    set_last_error_message(
+        "archead_forward_decode_noalloc: this head needs more scratch than the fixed 512 KiB array holds");
+    return ARCHEAD_ERR_UNSUPPORTED;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaSetDevice(pack->device);
+  void *base = nullptr;
+  if (e == cudaSuccess) e = scratch_address(pack->device, &base);
+  if (e != cudaSuccess) {
+    set_last_error_message(cudaGetErrorString(e));
+    return ARCHEAD_ERR_CUDA;
+  }
+  char *scratch = static_cast<char *>(base);
+  int *counters = reinterpret_cast<int *>(scratch);
+  float *partial = reinterpret_cast<float *>(scratch + kNoallocCounterBytes);
+  uint32_t *ts = reinterpret_cast<uint32_t *>(scratch + kNoallocCounterBytes + partial_bytes);
+
+  // The counters are the only state that must start at zero.
+  e = cudaMemsetAsync(counters, 0, (size_t)pairs * sizeof(int), s);
+
+  PrepassParams pp{};
+  pp.x = static_cast<const uint16_t *>(x);
+  pp.q_v = pack->q_v;
+  pp.q_b = pack->q_b;
+  pp.s_b = pack->s_b;
+  pp.s_u = pack->s_u;
+  pp.s_v = pack->s_v;
+  pp.M = (int)M;
+  pp.d = pack->d;
+  pp.g = pack->g;
+  pp.rc = pack->rc;
+  pp.rr = pack->rr;
+  pp.rcp = pack->rcp;
+  pp.rrp = pack->rrp;
+  pp.lr = pack->lr;
+  pp.partial = partial;
+  pp.counters = counters;
+  pp.ts = ts;
+  pp.T = nullptr;
+  if (e == cudaSuccess) e = launch_prepass(pp, s, nullptr);  // no profiling events on this path
+
+  DecodeParams dp{};
+  dp.codes = pack->codes;
+  dp.scales = pack->scales;
+  dp.lr_codes = pack->lr_codes;
+  dp.s_a = pack->s_a;
+  dp.x = static_cast<const uint16_t *>(x);
+  dp.ts = ts;
+  dp.V = pack->V;
+  dp.num_tiles = pack->num_tiles;
+  dp.d = pack->d;
+  dp.d_pad = pack->d_pad;
+  dp.G_pad = pack->G_pad;
+  dp.g = pack->g;
+  dp.nls = pack->nls;
+  dp.nls_core = pack->nls_core;
+  dp.M = (int)M;
+  dp.m0 = 0;
+  dp.NT = M > 8 ? 2 : 1;
+  dp.out = logits;
+  dp.out_fp32 = out_dtype == ARCHEAD_OUT_FP32;
+  dp.M_total = (int)M;
+  dp.err = pack->err;
+  dp.wait_budget = pack->wait_budget;
+  const int units = decode_num_units(pack);
+  if (e == cudaSuccess) e = launch_decode(dp, units < pack->sm_count ? units : pack->sm_count, s, pack->lr > 0);
+  if (e != cudaSuccess) {
+    set_last_error_message(cudaGetErrorString(e));
+    return ARCHEAD_ERR_CUDA;
+  }
+  return ARCHEAD_OK;
+}

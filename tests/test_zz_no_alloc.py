@@ -1,0 +1,97 @@
+"""archead_forward_decode_noalloc: the decode forward for callers that must
+not allocate device memory while they run the head (memory reserved up front,
+graph capture under a pool that forbids new allocations, latency-critical
+loops).  Its scratch is a fixed 512 KiB array inside the library instead of the
+pack's cudaMalloc-grown workspace.
+
+The test compares it, through the C ABI, with archead_forward on the same
+inputs, on two calls in a row (the second call finds the first call's data in
+the shared array).  This file is collected last on purpose.
+"""
+
+import zlib
+
+import numpy as np
+import pytest
+
+from paper_2608_02703_gb300 import archead
+from synth import HeadShape, make_head, make_hidden
+from tests import gpu_util as gu
+
+pytestmark = pytest.mark.gpu
+
+SHAPES = [
+    HeadShape(V=1000, d=256, core_rank=16, corr_rank=8, group_size=64),
+    HeadShape(V=4096, d=512, core_rank=64, corr_rank=16, group_size=64),
+    HeadShape(V=700, d=320, core_rank=24, corr_rank=40, group_size=32),
+]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _build():
+    from paper_2608_02703_gb300.build import build
+
+    build()
+
+
+def _run_noalloc(pack, x_bits, out_dtype):
+    import torch
+
+    M = x_bits.shape[0]
+    dt = torch.float32 if out_dtype == archead.OUT_FP32 else torch.bfloat16
+    y = torch.full((M, pack.shape.V), float("nan"), dtype=dt, device="cuda")
+    archead.archead_forward_decode_noalloc(pack, gu.to_dev(x_bits), M, y, out_dtype)
+    assert archead.archead_sync_status(pack) == archead.OK
+    return y.float().cpu().numpy().astype(np.float64)
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=lambda s: f"V{s.V}_d{s.d}_g{s.group_size}")
+@pytest.mark.parametrize("out_dtype", [archead.OUT_FP32, archead.OUT_BF16])
+def test_noalloc_matches_forward_on_two_calls_in_a_row(shape, out_dtype):
+    head = make_head(shape, seed=zlib.crc32(repr(shape).encode()) % 1000)
+    pack = archead.archead_pack_create(head, shape)
+    try:
+        for M, seed in ((7, 1), (16, 2), (1, 3)):
+            x = make_hidden(shape.d, M, seed=seed)
+            ref = gu.forward(pack, x, out_dtype, archead.PATH_DECODE)
+            first = _run_noalloc(pack, x, out_dtype)
+            second = _run_noalloc(pack, x, out_dtype)
+            for got in (first, second):
+                gu.check_logits(got, ref, bf16=False, where=f"noalloc M={M}")
+            assert np.array_equal(first, second)
+    finally:
+        pack.close()
+
+
+def test_noalloc_rejects_more_than_16_tokens():
+    import torch
+
+    shape = SHAPES[0]
+    pack = archead.archead_pack_create(make_head(shape, seed=5), shape)
+    try:
+        x = gu.to_dev(make_hidden(shape.d, 17, seed=5))
+        y = torch.empty((17, shape.V), dtype=torch.float32, device="cuda")
+        with pytest.raises(archead.ArcheadError) as exc:
+            archead.archead_forward_decode_noalloc(pack, x, 17, y, archead.OUT_FP32)
+        assert exc.value.status == archead.ERR_UNSUPPORTED
+        assert "at most 16" in str(exc.value)
+    finally:
+        pack.close()
+
+
+def test_noalloc_rejects_heads_needing_more_scratch():
+    import torch
+
+    # Ranks 256 + 256 at d = 4096: the pre-pass partial sums alone take
+    # 16 column blocks x 16 splits x 2 KB = 512 KiB, beyond the fixed array.
+    shape = HeadShape(V=128, d=4096, core_rank=256, corr_rank=256, group_size=128)
+    pack = archead.archead_pack_create(make_head(shape, seed=6), shape)
+    try:
+        x = gu.to_dev(make_hidden(shape.d, 1, seed=6))
+        y = torch.empty((1, shape.V), dtype=torch.float32, device="cuda")
+        with pytest.raises(archead.ArcheadError) as exc:
+            archead.archead_forward_decode_noalloc(pack, x, 1, y, archead.OUT_FP32)
+        assert exc.value.status == archead.ERR_UNSUPPORTED
+        assert "512 KiB" in str(exc.value)
+    finally:
+        pack.close()
