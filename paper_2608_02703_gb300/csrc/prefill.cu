@@ -26,7 +26,7 @@
 namespace archead {
 
 constexpr int kPfN = 256;                         // tokens per tile
-constexpr int kPfStages = 3;
+constexpr int kPfStages = 4;
 constexpr int kPfABytes = kTileRows * 64 * 2;     // 16 KB
 constexpr int kPfBBytes = kPfN * 64 * 2;          // 32 KB
 constexpr int kPfCodeBytes = 4 * kLrStepBytes;    // 8 KB (4 KB of INT4 or 4 low-rank steps)
@@ -234,8 +234,8 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
         int blk = 0, in_blk = 0;
         int blk_len = bp.G_pad > 0 ? bp.gsub : (bp.core_sub > 0 ? bp.core_sub : bp.corr_sub);
         for (int e = 0; e < KS; ++e) {
+          // The converters arrive on a_full only after the stage's TMA bytes landed.
           if (!mbar_wait(&a_full[s], ph, p.wait_budget, abort_flag, p.err)) goto done;
-          if (!mbar_wait(&full[s], ph, p.wait_budget, abort_flag, p.err)) goto done;
           tc_fence_after();
           const uint32_t a_base = smem_u32(smem + s * kPfStageBytes);
           const uint32_t b_base = a_base + kPfABytes;
