@@ -167,6 +167,37 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, int64_
   }
 }
 
+// True in exactly one lane of a converged warp (elect.sync).  Guarding the
+// single-thread issue of tcgen05 / TMA instructions with it, instead of a
+// test on the lane index, keeps the issuing code warp-uniform.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t pred = 0;
+  asm volatile(
+      "{\n .reg .b32 r;\n .reg .pred p;\n elect.sync r|p, 0xffffffff;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(pred));
+  return pred != 0;
+}
+
+// mbar_wait for a whole converged warp: every lane calls it and every lane
+// gets the same answer (the decisions are warp votes), so the code after a
+// wait stays warp-uniform.  Same bound and error reporting as mbar_wait.
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t *bar, uint32_t parity, int64_t budget,
+                                               volatile int *abort_flag, int *err) {
+  if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
+    if (__any_sync(0xffffffffu, abort_flag != nullptr && *abort_flag)) return false;
+    if (__any_sync(0xffffffffu, clock64() - t0 > budget)) {
+      if (elect_one()) {
+        atomicOr(err, kErrWaitTimeout);
+        if (abort_flag != nullptr) *abort_flag = 1;
+      }
+      return false;
+    }
+  }
+}
+
 // Global -> shared bulk copy completing on an mbarrier (size multiple of 16,
 // both addresses 16-byte aligned).
 __device__ __forceinline__ void bulk_g2s(void *dst_smem, const void *src_gmem, uint32_t bytes, uint64_t *bar) {

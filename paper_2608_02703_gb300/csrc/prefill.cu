@@ -179,6 +179,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  bool mma_leader = false;  // the lane of warp 1 that issues the MMAs
 
   // Registers are rebalanced between warpgroups (launch: 512 x 128): the
   // producer/MMA warpgroup and the converters keep 56 each, the two promotion
@@ -189,18 +190,21 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     asm volatile("setmaxnreg.dec.sync.aligned.u32 56;\n" ::: "memory");
   if (warp == 0) {
     // ------------------------------ producer ------------------------------
-    if (lane == 0) {
+    // The whole warp runs the loop (uniform waits); one elected lane issues.
+    {
+      const bool leader = elect_one();
       int s = 0;
       uint32_t ph = 0;
       for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
         const int vt = t / p.num_mt, mt = t % p.num_mt;
         const int m0 = mt * kPfN;
         for (int e = 0; e < KS; ++e) {
-          if (!mbar_wait(&empty[s], ph ^ 1, p.wait_budget, abort_flag, p.err)) goto done;
+          if (!mbar_wait_warp(&empty[s], ph ^ 1, p.wait_budget, abort_flag, p.err)) goto done;
           uint8_t *st = smem + s * kPfStageBytes;
           uint8_t *bdst = st + kPfABytes;
           uint8_t *cdst = bdst + kPfBBytes;
-          if (e < KC) {
+          if (!leader) {
+          } else if (e < KC) {
             mbar_arrive_expect_tx(&full[s], kPfBBytes + kChunkBytes);
             tma_load_2d(bdst, &p.tmap_x, e * 64, m0, &full[s]);
             tma_load_2d(bdst + kPfBBytes / 2, &p.tmap_x, e * 64, m0 + 128, &full[s]);
@@ -220,13 +224,22 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
             }
           }
           if (++s == kPfStages) s = 0, ph ^= 1;
+          __syncwarp();
         }
       }
     }
   } else if (warp == 1) {
     // ------------------------------ MMA issuer ------------------------------
-    if (lane == 0) {
+    // As for the producer: the warp runs the loop, one elected lane issues.
+    // Keeping the loop warp-uniform (votes on every wait, elect.sync for the
+    // issuing lane) is what lets the MMAs issue back to back.
+    {
+      const bool leader = elect_one();
+      mma_leader = leader;
       constexpr uint32_t idesc = idesc_bf16(128, kPfN);
+      const uint64_t desc0 = smem_desc_sw128(smem_u32(smem));
+      constexpr uint32_t kStageDesc = kPfStageBytes >> 4;  // descriptor address step of one stage
+      constexpr uint32_t kBDesc = kPfABytes >> 4;           // A -> B within a stage
       int s = 0;
       uint32_t ph = 0;
       int bcount = 0;  // accumulator blocks started so far
@@ -235,28 +248,31 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
         int blk_len = bp.G_pad > 0 ? bp.gsub : (bp.core_sub > 0 ? bp.core_sub : bp.corr_sub);
         for (int e = 0; e < KS; ++e) {
           // The converters arrive on a_full only after the stage's TMA bytes landed.
-          if (!mbar_wait(&a_full[s], ph, p.wait_budget, abort_flag, p.err)) goto done;
+          if (!mbar_wait_warp(&a_full[s], ph, p.wait_budget, abort_flag, p.err)) goto done;
           tc_fence_after();
-          const uint32_t a_base = smem_u32(smem + s * kPfStageBytes);
-          const uint32_t b_base = a_base + kPfABytes;
+          const uint64_t ad = desc0 + (uint64_t)(s * kStageDesc);
+          const uint64_t bd = ad + kBDesc;
+#pragma unroll
           for (int q = 0; q < 4; ++q) {
             const int buf = bcount & 1;
             if (in_blk == 0) {
-              if (!mbar_wait(&acc_empty[buf], ((bcount >> 1) & 1) ^ 1, p.wait_budget, abort_flag, p.err)) goto done;
+              if (!mbar_wait_warp(&acc_empty[buf], ((bcount >> 1) & 1) ^ 1, p.wait_budget, abort_flag, p.err))
+                goto done;
               tc_fence_after();
             }
-            tc_mma(tmem_base + buf * kPfN, smem_desc_sw128(a_base + q * 32), smem_desc_sw128(b_base + q * 32), idesc,
-                   in_blk > 0);
+            // +2 per 16-wide k step: 32 bytes in the descriptor's 16-byte address units.
+            if (leader) tc_mma(tmem_base + buf * kPfN, ad + 2 * q, bd + 2 * q, idesc, in_blk > 0);
             if (++in_blk == blk_len) {
-              tc_commit(&acc_full[buf]);
+              if (leader) tc_commit(&acc_full[buf]);
               ++bcount;
               ++blk;
               in_blk = 0;
               blk_len = blk < bp.G_pad ? bp.gsub : (blk == bp.G_pad && bp.core_sub > 0 ? bp.core_sub : bp.corr_sub);
             }
           }
-          tc_commit(&empty[s]);
+          if (leader) tc_commit(&empty[s]);
           if (++s == kPfStages) s = 0, ph ^= 1;
+          __syncwarp();
         }
       }
     }
@@ -270,7 +286,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     uint32_t ph = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
       for (int e = 0; e < KS; ++e) {
-        if (!mbar_wait(&full[s], ph, p.wait_budget, abort_flag, p.err)) goto done;
+        if (!mbar_wait_warp(&full[s], ph, p.wait_budget, abort_flag, p.err)) goto done;
         uint8_t *a_tile = smem + s * kPfStageBytes;
         const uint8_t *codes = a_tile + kPfABytes + kPfBBytes;
 #pragma unroll
@@ -333,7 +349,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
         else if (b == bp.G_pad && bp.core_sub > 0) f = 1.f;
         else f = fp16_bits_to_f32(p.s_a[row]);
         const int buf = bcount & 1;
-        if (!mbar_wait(&acc_full[buf], (bcount >> 1) & 1, p.wait_budget, abort_flag, p.err)) goto done;
+        if (!mbar_wait_warp(&acc_full[buf], (bcount >> 1) & 1, p.wait_budget, abort_flag, p.err)) goto done;
         tc_fence_after();
         const uint32_t taddr = tmem_base + ((uint32_t)(lg * 32) << 16) + buf * kPfN + ch * 128;
 #pragma unroll
@@ -384,7 +400,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     }
   }
 done:
-  if (warp == 1 && lane == 0) {
+  if (warp == 1 && mma_leader) {
     // Every MMA this thread issued has completed before TMEM is released.
     tc_commit(drain);
     mbar_wait(drain, 0, p.wait_budget, nullptr, p.err);
@@ -409,7 +425,7 @@ static EncodeTiledFn encode_fn() {
   if (!fn) {
     void *ptr = nullptr;
     cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &ptr, cudaEnableDefault, &q) == cudaSuccess &&
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
       fn = reinterpret_cast<EncodeTiledFn>(ptr);
   }
