@@ -107,6 +107,22 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// d0 += a * b0 and d1 += a * b1 as one packed fp32x2 FMA (round to nearest).
+__device__ __forceinline__ void fma2(float &d0, float &d1, float a, float b0, float b1) {
+  asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %2};\n mov.b64 rb, {%3, %4};\n mov.b64 rd, {%0, %1};\n"
+      " fma.rn.f32x2 rd, ra, rb, rd;\n mov.b64 {%0, %1}, rd;\n}\n"
+      : "+f"(d0), "+f"(d1)
+      : "f"(a), "f"(b0), "f"(b1));
+}
+
+// One step of the log-sum-exp merge: (m, s) of two disjoint sets -> of their union.
+__device__ __forceinline__ void lse_pair_merge(float am, float as, float bm, float bs, float &m, float &s) {
+  const float mx = fmaxf(am, bm), mn = fminf(am, bm);
+  const float e = mn == -INFINITY ? 0.f : __expf(mn - mx);
+  s = am >= bm ? fmaf(bs, e, as) : fmaf(as, e, bs);
+  m = mx;
+}
+
 // Shared-memory matrix descriptor: K-major operand in the 128-byte swizzle
 // layout (8-row groups of 128-byte rows, 1024 bytes apart).
 __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
@@ -357,7 +373,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
           float v[32];
           tmem_ld32(taddr + c * 32, v);
 #pragma unroll
-          for (int i = 0; i < 32; ++i) acc[c * 32 + i] = fmaf(f, v[i], acc[c * 32 + i]);
+          for (int i = 0; i < 32; i += 2) fma2(acc[c * 32 + i], acc[c * 32 + i + 1], f, v[i], v[i + 1]);
         }
         tc_fence_before();
         __syncwarp();
@@ -380,21 +396,61 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
           }
         }
       } else {
-        const bool valid_row = row < p.V;
+        // Target logits first: a token whose target is one of this warp's 32
+        // rows takes its value from the owning lane (rare: about one token in
+        // 37 per warp and tile, so the slow path is a warp-uniform branch).
+        const int64_t rowbase = row - lane;
+        int tg[4];
+        bool hit = false;
 #pragma unroll
-        for (int i = 0; i < 128; ++i) {
-          const int m = m0 + i;
-          const float v = valid_row ? acc[i] : -INFINITY;
-          LsePair lp{v, valid_row ? 1.f : 0.f};
+        for (int j = 0; j < 4; ++j) {
+          const int m = m0 + 4 * lane + j;
+          tg[j] = m < p.M ? p.targets[m] : -1;
+          hit |= tg[j] >= rowbase && tg[j] < rowbase + 32;
+        }
+        if (__any_sync(0xffffffffu, hit)) {
 #pragma unroll
-          for (int off = 1; off < 32; off <<= 1) {
-            LsePair o{__shfl_xor_sync(0xffffffffu, lp.m, off), __shfl_xor_sync(0xffffffffu, lp.s, off)};
-            lp = lse_merge(lp, o);
+          for (int k = 0; k < 128; ++k) {
+            const int tk = __shfl_sync(0xffffffffu, tg[k & 3], k >> 2);
+            const float val = __shfl_sync(0xffffffffu, acc[k], (int)((tk - rowbase) & 31));
+            if (lane == (k >> 2) && tk >= rowbase && tk < rowbase + 32) p.ce_tlogit[m0 + k] = val;
           }
-          if (m < p.M) {
-            if (lane == 0) p.ce_part[((int64_t)vt * 4 + lg) * p.M + m] = make_float2(lp.m, lp.s);
-            if (valid_row && p.targets[m] == row) p.ce_tlogit[m] = v;
+        }
+        // (max, sum of exp) over the warp's 32 rows for each of the 128
+        // tokens, by a butterfly that halves the token set per step: in the
+        // step with lane offset o the lane with bit o set keeps the upper
+        // half and merges the partner's copy of it.  After the five steps
+        // lane L holds tokens 4L..4L+3.  Maxima live in acc[0..63], sums in
+        // acc[64..127]; rows past V enter as -inf.
+        if (row >= p.V) {
+#pragma unroll
+          for (int i = 0; i < 128; ++i) acc[i] = -INFINITY;
+        }
+        {
+          const bool up = lane & 16;
+#pragma unroll
+          for (int j = 0; j < 64; ++j) {
+            const float keep = up ? acc[j + 64] : acc[j];
+            const float give = up ? acc[j] : acc[j + 64];
+            const float recv = __shfl_xor_sync(0xffffffffu, give, 16);
+            lse_pair_merge(keep, 1.f, recv, 1.f, acc[j], acc[64 + j]);
           }
+        }
+#pragma unroll
+        for (int n = 64, o = 8; n > 4; n >>= 1, o >>= 1) {
+          const bool up = lane & o;
+#pragma unroll
+          for (int j = 0; j < n / 2; ++j) {
+            const float km = up ? acc[j + n / 2] : acc[j], ks = up ? acc[64 + j + n / 2] : acc[64 + j];
+            const float gm = up ? acc[j] : acc[j + n / 2], gs = up ? acc[64 + j] : acc[64 + j + n / 2];
+            const float rm = __shfl_xor_sync(0xffffffffu, gm, o), rs = __shfl_xor_sync(0xffffffffu, gs, o);
+            lse_pair_merge(km, ks, rm, rs, acc[j], acc[64 + j]);
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int m = m0 + 4 * lane + j;
+          if (m < p.M) p.ce_part[((int64_t)vt * 4 + lg) * p.M + m] = make_float2(acc[j], acc[64 + j]);
         }
       }
     }
