@@ -383,16 +383,17 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
       // Epilogue: columns are tokens m0 + i, this thread's row is `row`.
       if (kMode == 0) {
         if (row < p.V) {
+          const int mcount = p.M - m0 < 128 ? p.M - m0 : 128;  // tokens of this column half inside M
+          if (p.out_fp32) {
+            float *o = reinterpret_cast<float *>(p.out) + (int64_t)m0 * p.V + row;
 #pragma unroll
-          for (int i = 0; i < 128; ++i) {
-            const int m = m0 + i;
-            if (m < p.M) {
-              const int64_t o = (int64_t)m * p.V + row;
-              if (p.out_fp32)
-                reinterpret_cast<float *>(p.out)[o] = acc[i];
-              else
-                reinterpret_cast<__nv_bfloat16 *>(p.out)[o] = __float2bfloat16_rn(acc[i]);
-            }
+            for (int i = 0; i < 128; ++i, o += p.V)
+              if (i < mcount) *o = acc[i];
+          } else {
+            __nv_bfloat16 *o = reinterpret_cast<__nv_bfloat16 *>(p.out) + (int64_t)m0 * p.V + row;
+#pragma unroll
+            for (int i = 0; i < 128; ++i, o += p.V)
+              if (i < mcount) *o = __float2bfloat16_rn(acc[i]);
           }
         }
       } else {
