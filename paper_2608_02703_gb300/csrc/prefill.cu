@@ -198,12 +198,13 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   bool mma_leader = false;  // the lane of warp 1 that issues the MMAs
 
   // Registers are rebalanced between warpgroups (launch: 512 x 128): the
-  // producer/MMA warpgroup and the converters keep 56 each, the two promotion
-  // warpgroups get 200 each (128 fp32 accumulators per thread).
-  // 4*32*(56 + 56) + 8*32*200 = 65536.  Each role's code follows its own
-  // setmaxnreg so that the compiler allocates within that budget.
+  // producer/MMA warpgroup and the converters keep 88 each, the two promotion
+  // warpgroups get 168 each (128 fp32 accumulators per thread):
+  // 4*32*(88 + 88) + 8*32*168 = 65536.  Each role's code follows its own
+  // setmaxnreg so that the compiler allocates within that budget; this split
+  // is the one that compiles without spills.
   if (warp < 4) {
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 56;\n" ::: "memory");
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 88;\n" ::: "memory");
   if (warp == 0) {
     // ------------------------------ producer ------------------------------
     // The whole warp runs the loop (uniform waits); one elected lane issues.
@@ -295,7 +296,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   }
   } else if (warp < 8) {
     // ------------------------------ converters ------------------------------
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 56;\n" ::: "memory");
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 88;\n" ::: "memory");
     const int cw = warp - 4;
     const int gq = lane >> 2, cq = lane & 3;
     int s = 0;
@@ -345,7 +346,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     }
   } else {
     // ------------------------------ promotion + epilogue ------------------------------
-    asm volatile("setmaxnreg.inc.sync.aligned.u32 200;\n" ::: "memory");
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 168;\n" ::: "memory");
     const int pw = warp - 8;
     const int lg = pw & 3;            // TMEM lane group (rows 32*lg .. 32*lg+31)
     const int ch = pw >> 2;           // column half (tokens 128*ch .. 128*ch+127)
