@@ -41,8 +41,8 @@ cudaError_t dev_alloc(archead_pack *p, T **ptr, size_t bytes) {
 
 void free_pack(archead_pack *p) {
   if (!p) return;
-  void *bufs[] = {p->codes, p->scales, p->lr_codes, p->s_a, p->q_v, p->q_b, p->s_u,
-                  p->s_v,   p->s_b,    p->err,      p->ws,  p->xh_dev, p->yh_dev, p->counters};
+  void *bufs[] = {p->codes, p->scales, p->lr_codes, p->s_a,    p->q_v,    p->q_b,   p->lr_t, p->s_u,
+                  p->s_v,   p->s_b,    p->err,      p->ws,     p->xh_dev, p->yh_dev, p->counters};
   for (void *b : bufs)
     if (b) cudaFree(b);
   for (auto &t : p->timers)
@@ -223,7 +223,6 @@ archead_status run_prefill(archead_pack *p, const void *x, int64_t M, void *out,
                            const int32_t *targets, float *ce, cudaStream_t s) {
   const bool ce_mode = out == nullptr;
   Carve c;
-  const size_t partial_off = c.take(prepass_partial_bytes((int)M, p->lr, p->d));
   const size_t t_off = c.take((size_t)M * std::max(2 * p->lr, 64) * 2);
   size_t ce_part_off = 0, tlogit_off = 0;
   if (ce_mode) {
@@ -231,13 +230,10 @@ archead_status run_prefill(archead_pack *p, const void *x, int64_t M, void *out,
     tlogit_off = c.take((size_t)M * sizeof(float));
   }
   AH_CUDA(ensure_workspace(p, c.off, s));
-  AH_CUDA(ensure_counters(p, prepass_pairs((int)M, p->lr), s));
   PrepassParams pp = prepass_params(p, x, M);
-  pp.partial = at<float>(p->ws, partial_off);
-  pp.counters = p->counters;
   pp.ts = nullptr;
   pp.T = at<uint16_t>(p->ws, t_off);
-  AH_CUDA(launch_prepass(pp, s, p));
+  AH_CUDA(launch_prepass_t(pp, p->lr_t, p->d_pad, s, p));
   float2 *ce_part = ce_mode ? at<float2>(p->ws, ce_part_off) : nullptr;
   float *tlogit = ce_mode ? at<float>(p->ws, tlogit_off) : nullptr;
   cudaEvent_t ev = nullptr;
@@ -355,6 +351,7 @@ archead_status archead_pack_create(const archead_desc *desc, void *stream, arche
   if ((e = dev_alloc(p, &p->s_a, (size_t)p->V_pad * 2)) != cudaSuccess) return fail(e);
   if ((e = dev_alloc(p, &p->q_v, (size_t)d * rc)) != cudaSuccess) return fail(e);
   if ((e = dev_alloc(p, &p->q_b, (size_t)d * rr)) != cudaSuccess) return fail(e);
+  if ((e = dev_alloc(p, &p->lr_t, (size_t)p->lr * p->d_pad * 2)) != cudaSuccess) return fail(e);
   if ((e = dev_alloc(p, &p->s_u, (size_t)rc * 2)) != cudaSuccess) return fail(e);
   if ((e = dev_alloc(p, &p->s_v, (size_t)rc * 2)) != cudaSuccess) return fail(e);
   if ((e = dev_alloc(p, &p->s_b, G * rr * 2)) != cudaSuccess) return fail(e);

@@ -102,6 +102,7 @@ struct archead_pack {
   uint8_t *lr_codes = nullptr;
   uint16_t *s_a = nullptr;
   int8_t *q_v = nullptr, *q_b = nullptr;
+  uint16_t *lr_t = nullptr;  // [lr][d_pad] bf16: extended column kk of [q_v | q_b] (zero padded), k fastest
   uint16_t *s_u = nullptr, *s_v = nullptr, *s_b = nullptr;
   int *err = nullptr;
   int64_t owned_bytes = 0;
@@ -128,6 +129,9 @@ cudaError_t launch_debug_dequant(const archead_pack *p, int comp, int64_t row0, 
                                  cudaStream_t s);
 cudaError_t launch_prepass(const PrepassParams &pp, cudaStream_t s, archead_pack *p);
 int prepass_pairs(int M, int lr);
+// Tensor-core pre-pass for many tokens: writes the prefill operand T only.
+cudaError_t launch_prepass_t(const PrepassParams &pp, const uint16_t *lr_t, int d_pad, cudaStream_t s,
+                             archead_pack *pk);
 size_t prepass_smem(int M);  // dynamic shared memory of one pre-pass block
 size_t prepass_partial_bytes(int M, int lr, int d);
 // pdl: launch as a programmatic dependent of the immediately preceding pre-pass grid.

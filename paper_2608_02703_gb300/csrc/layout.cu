@@ -80,6 +80,25 @@ __global__ void build_row_scales_kernel(const uint16_t *__restrict__ src, uint16
     dst[i] = (src != nullptr && i < V) ? src[i] : (uint16_t)0;
 }
 
+// The pre-pass operand of the prefill path, transposed to [extended column][k]
+// and widened to bf16 (the int8 codes are exact in bf16).
+__global__ void build_lr_t_kernel(const int8_t *__restrict__ q_v, const int8_t *__restrict__ q_b,
+                                  uint16_t *__restrict__ dst, int d, int d_pad, int rc, int rr, int rcp, int lr) {
+  const int64_t total = (int64_t)lr * d_pad;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const int kk = (int)(i / d_pad), k = (int)(i % d_pad);
+    int code = 0;
+    if (k < d) {
+      if (kk < rcp) {
+        if (kk < rc) code = q_v[(int64_t)k * rc + kk];
+      } else if (kk - rcp < rr) {
+        code = q_b[(int64_t)k * rr + (kk - rcp)];
+      }
+    }
+    dst[i] = __bfloat16_as_ushort(__int2bfloat16_rn(code));
+  }
+}
+
 cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, const uint16_t *res_scales,
                                  const int8_t *core_u, const int8_t *corr_a, const uint16_t *corr_a_scale,
                                  cudaStream_t s) {
@@ -90,6 +109,8 @@ cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, cons
     build_lr_codes_kernel<<<p->num_tiles * p->nls, 256, 0, s>>>(core_u, corr_a, p->lr_codes, p->V, p->rc, p->rr,
                                                                  p->rcp, p->nls);
   build_row_scales_kernel<<<256, 256, 0, s>>>(p->rr > 0 ? corr_a_scale : nullptr, p->s_a, p->V, p->V_pad);
+  if (p->lr > 0)
+    build_lr_t_kernel<<<256, 256, 0, s>>>(p->q_v, p->q_b, p->lr_t, p->d, p->d_pad, p->rc, p->rr, p->rcp, p->lr);
   return cudaGetLastError();
 }
 

@@ -154,6 +154,162 @@ __global__ void __launch_bounds__(256) prepass_kernel(PrepassParams p) {
   if (threadIdx.x == 0) p.counters[pair] = 0;  // ready for the next call
 }
 
+// ---------------------------------------------------------------------------
+// Tensor-core pre-pass for many tokens (prefill).  Same t as above, written
+// only to the row-major operand T.  Block: 64 tokens x 32 extended columns,
+// the whole of d (no split, so no partial sums and no counters); warp w takes
+// tokens 16w..16w+15 with mma.sync m16n8k16 (bf16 in, fp32 accumulate) over
+// 128-wide chunks of d staged in shared memory by cp.async (double buffer).
+// A = x rows, B = lr_t rows (the extended column's int8 codes as bf16).  In
+// a correction block the accumulators are scaled by s_b at the end of every
+// quantisation group and added to running sums; a core block scales once by
+// s_u s_v at the end.
+// ---------------------------------------------------------------------------
+constexpr int kPtTok = 64;
+constexpr int kPtCols = 32;
+constexpr int kPtK = 128;
+constexpr int kPtStride = kPtK + 8;  // bf16 per staged row: conflict-free fragment loads
+constexpr int kPtSmem = 2 * (kPtTok + kPtCols) * kPtStride * 2;
+
+__device__ __forceinline__ void cp_async16(void *dst, const void *src, bool valid) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(smem_u32(dst)), "l"(src),
+               "r"(valid ? 16 : 0)
+               : "memory");
+}
+
+__global__ void __launch_bounds__(128) prepass_t_kernel(PrepassParams p, const uint16_t *__restrict__ lr_t,
+                                                        int d_pad) {
+  extern __shared__ __align__(16) uint16_t pt_smem[];
+  uint16_t *xs = pt_smem;                            // [2][64][kPtStride]
+  uint16_t *bs = pt_smem + 2 * kPtTok * kPtStride;   // [2][32][kPtStride]
+  const int c0 = blockIdx.x * kPtCols;
+  const int m0 = blockIdx.y * kPtTok;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int gq = lane >> 2, cq = lane & 3;
+  const bool core = c0 < p.rcp;  // a 32-column block never straddles the core/correction boundary
+  const int nchunks = d_pad / kPtK;
+
+  auto stage = [&](int kc, int buf) {
+    const int k0 = kc * kPtK;
+    // x: 64 rows x 16 pieces of 16 bytes; tokens past M and k past d read as zero.
+    for (int i = threadIdx.x; i < kPtTok * 16; i += blockDim.x) {
+      const int r = i >> 4, c = i & 15;
+      const int m = m0 + r, k = k0 + c * 8;
+      const bool ok = m < p.M && k < p.d;
+      cp_async16(xs + (buf * kPtTok + r) * kPtStride + c * 8, ok ? p.x + (int64_t)m * p.d + k : p.x, ok);
+    }
+    for (int i = threadIdx.x; i < kPtCols * 16; i += blockDim.x) {
+      const int r = i >> 4, c = i & 15;
+      cp_async16(bs + (buf * kPtCols + r) * kPtStride + c * 8, lr_t + (int64_t)(c0 + r) * d_pad + k0 + c * 8, true);
+    }
+    asm volatile("cp.async.commit_group;\n" ::: "memory");
+  };
+
+  float acc[4][4], run[4][4];
+#pragma unroll
+  for (int n = 0; n < 4; ++n)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) acc[n][i] = run[n][i] = 0.f;
+
+  stage(0, 0);
+  for (int kc = 0; kc < nchunks; ++kc) {
+    const int buf = kc & 1;
+    if (kc + 1 < nchunks) {
+      stage(kc + 1, buf ^ 1);
+      asm volatile("cp.async.wait_group 1;\n" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;\n" ::: "memory");
+    }
+    __syncthreads();
+    const uint16_t *xa = xs + (buf * kPtTok + warp * 16) * kPtStride;
+    const uint16_t *xb = bs + buf * kPtCols * kPtStride;
+#pragma unroll
+    for (int ks = 0; ks < kPtK / 16; ++ks) {
+      const int kb = ks * 16 + 2 * cq;
+      uint32_t a[4];
+      a[0] = *reinterpret_cast<const uint32_t *>(xa + gq * kPtStride + kb);
+      a[1] = *reinterpret_cast<const uint32_t *>(xa + (gq + 8) * kPtStride + kb);
+      a[2] = *reinterpret_cast<const uint32_t *>(xa + gq * kPtStride + kb + 8);
+      a[3] = *reinterpret_cast<const uint32_t *>(xa + (gq + 8) * kPtStride + kb + 8);
+#pragma unroll
+      for (int n = 0; n < 4; ++n) {
+        const uint16_t *br = xb + (n * 8 + gq) * kPtStride + kb;
+        mma_bf16_16816(acc[n], a, *reinterpret_cast<const uint32_t *>(br), *reinterpret_cast<const uint32_t *>(br + 8));
+      }
+      // End of a quantisation group of the correction factor: apply s_b.
+      const int kend = kc * kPtK + ks * 16 + 16;
+      if (!core && kend % p.g == 0) {
+        const int grp = kend / p.g - 1;
+        if (grp < p.d / p.g) {
+#pragma unroll
+          for (int n = 0; n < 4; ++n) {
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const int j = c0 - p.rcp + n * 8 + 2 * cq + h;
+              const float sb = j < p.rr ? fp16_bits_to_f32(p.s_b[(int64_t)grp * p.rr + j]) : 0.f;
+              run[n][h] = fmaf(sb, acc[n][h], run[n][h]);
+              run[n][2 + h] = fmaf(sb, acc[n][2 + h], run[n][2 + h]);
+            }
+          }
+        }
+#pragma unroll
+        for (int n = 0; n < 4; ++n)
+#pragma unroll
+          for (int i = 0; i < 4; ++i) acc[n][i] = 0.f;
+      }
+    }
+    __syncthreads();  // the buffer is restaged two chunks later
+  }
+
+  // t for (token, column) pairs of this lane, then the bf16 hi/lo split.
+#pragma unroll
+  for (int n = 0; n < 4; ++n) {
+#pragma unroll
+    for (int rh = 0; rh < 2; ++rh) {
+      const int m = m0 + warp * 16 + gq + 8 * rh;
+      if (m >= p.M) continue;
+      uint32_t hi2 = 0, lo2 = 0;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int kk = c0 + n * 8 + 2 * cq + h;
+        float t;
+        if (core) {
+          t = kk < p.rc ? acc[n][2 * rh + h] * fp16_bits_to_f32(p.s_v[kk]) * fp16_bits_to_f32(p.s_u[kk]) : 0.f;
+        } else {
+          t = kk - p.rcp < p.rr ? run[n][2 * rh + h] : 0.f;
+        }
+        const uint16_t hi = f32_to_bf16_bits(t);
+        const uint16_t lo = f32_to_bf16_bits(t - bf16_lo(hi));
+        hi2 |= (uint32_t)hi << (16 * h);
+        lo2 |= (uint32_t)lo << (16 * h);
+      }
+      const int kk = c0 + n * 8 + 2 * cq;
+      uint16_t *row = p.T + (int64_t)m * (2 * p.lr);
+      const int hi_col = core ? kk : p.rcp + kk;                 // = 2 rcp + j for the correction
+      const int lo_col = core ? p.rcp + kk : p.rcp + p.rrp + kk;  // = 2 rcp + rrp + j
+      *reinterpret_cast<uint32_t *>(row + hi_col) = hi2;
+      *reinterpret_cast<uint32_t *>(row + lo_col) = lo2;
+    }
+  }
+}
+
+cudaError_t launch_prepass_t(const PrepassParams &pp, const uint16_t *lr_t, int d_pad, cudaStream_t s,
+                             archead_pack *pk) {
+  if (pp.lr == 0) return cudaSuccess;
+  cudaEvent_t ev = nullptr;
+  timer_begin(pk, "prepass", s, &ev);
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(prepass_t_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kPtSmem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  dim3 grid(pp.lr / kPtCols, (pp.M + kPtTok - 1) / kPtTok);
+  prepass_t_kernel<<<grid, 128, kPtSmem, s>>>(pp, lr_t, d_pad);
+  timer_end(pk, "prepass", s, ev);
+  return cudaGetLastError();
+}
+
 int prepass_pairs(int M, int lr) { return (lr / kPreCols) * ((M + kPreTok - 1) / kPreTok); }
 
 size_t prepass_partial_bytes(int M, int lr, int d) {
