@@ -159,7 +159,8 @@ __global__ void __launch_bounds__(256) prepass_kernel(PrepassParams p) {
 // only to the row-major operand T.  Block: 64 tokens x 32 extended columns,
 // the whole of d (no split, so no partial sums and no counters); warp w takes
 // tokens 16w..16w+15 with mma.sync m16n8k16 (bf16 in, fp32 accumulate) over
-// 128-wide chunks of d staged in shared memory by cp.async (double buffer).
+// 128-wide chunks of d staged in shared memory by cp.async (double buffer;
+// at 52 KB a block, four blocks share an SM and a 4096-token call is one wave).
 // A = x rows, B = lr_t rows (the extended column's int8 codes as bf16).  In
 // a correction block the accumulators are scaled by s_b at the end of every
 // quantisation group and added to running sums; a core block scales once by
@@ -169,7 +170,8 @@ constexpr int kPtTok = 64;
 constexpr int kPtCols = 32;
 constexpr int kPtK = 128;
 constexpr int kPtStride = kPtK + 8;  // bf16 per staged row: conflict-free fragment loads
-constexpr int kPtSmem = 2 * (kPtTok + kPtCols) * kPtStride * 2;
+constexpr int kPtStages = 2;
+constexpr int kPtSmem = kPtStages * (kPtTok + kPtCols) * kPtStride * 2;
 
 __device__ __forceinline__ void cp_async16(void *dst, const void *src, bool valid) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(smem_u32(dst)), "l"(src),
@@ -180,8 +182,8 @@ __device__ __forceinline__ void cp_async16(void *dst, const void *src, bool vali
 __global__ void __launch_bounds__(128) prepass_t_kernel(PrepassParams p, const uint16_t *__restrict__ lr_t,
                                                         int d_pad) {
   extern __shared__ __align__(16) uint16_t pt_smem[];
-  uint16_t *xs = pt_smem;                            // [2][64][kPtStride]
-  uint16_t *bs = pt_smem + 2 * kPtTok * kPtStride;   // [2][32][kPtStride]
+  uint16_t *xs = pt_smem;                                    // [stages][64][kPtStride]
+  uint16_t *bs = pt_smem + kPtStages * kPtTok * kPtStride;   // [stages][32][kPtStride]
   const int c0 = blockIdx.x * kPtCols;
   const int m0 = blockIdx.y * kPtTok;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -211,16 +213,21 @@ __global__ void __launch_bounds__(128) prepass_t_kernel(PrepassParams p, const u
 #pragma unroll
     for (int i = 0; i < 4; ++i) acc[n][i] = run[n][i] = 0.f;
 
-  stage(0, 0);
+  // Chunk c is cp.async group c: kPtStages-1 are committed up front and one
+  // (maybe empty) per iteration, after the wait, so when iteration kc waits
+  // the newest kPtStages-2 groups are later chunks and waiting for all but
+  // those completes chunk kc.  The barrier after the wait also guarantees
+  // that every warp is done with chunk kc-1, whose buffer is restaged next.
+  for (int kc = 0; kc < kPtStages - 1; ++kc) {
+    if (kc < nchunks) stage(kc, kc);
+    else asm volatile("cp.async.commit_group;\n" ::: "memory");
+  }
   for (int kc = 0; kc < nchunks; ++kc) {
-    const int buf = kc & 1;
-    if (kc + 1 < nchunks) {
-      stage(kc + 1, buf ^ 1);
-      asm volatile("cp.async.wait_group 1;\n" ::: "memory");
-    } else {
-      asm volatile("cp.async.wait_group 0;\n" ::: "memory");
-    }
+    const int buf = kc % kPtStages;
+    asm volatile("cp.async.wait_group %0;\n" ::"n"(kPtStages - 2) : "memory");
     __syncthreads();
+    if (kc + kPtStages - 1 < nchunks) stage(kc + kPtStages - 1, (kc + kPtStages - 1) % kPtStages);
+    else asm volatile("cp.async.commit_group;\n" ::: "memory");
     const uint16_t *xa = xs + (buf * kPtTok + warp * 16) * kPtStride;
     const uint16_t *xb = bs + buf * kPtCols * kPtStride;
 #pragma unroll
@@ -258,7 +265,6 @@ __global__ void __launch_bounds__(128) prepass_t_kernel(PrepassParams p, const u
           for (int i = 0; i < 4; ++i) acc[n][i] = 0.f;
       }
     }
-    __syncthreads();  // the buffer is restaged two chunks later
   }
 
   // t for (token, column) pairs of this lane, then the bf16 hi/lo split.
