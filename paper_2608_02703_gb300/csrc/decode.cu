@@ -151,10 +151,15 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
 
   if (warp == kDecWarps) {
     // ---------------- producer warp ----------------
-    if (lane != 0) return;
-    mbar_arrive_expect_tx(xbar, (uint32_t)(p.M * p.d * 2));
-    for (int m = 0; m < p.M; ++m)
-      bulk_g2s(smem + xs_off + (size_t)m * xrow * 2, p.x + (size_t)(p.m0 + m) * p.d, (uint32_t)(p.d * 2), xbar);
+    // The whole warp runs the loop (voted waits keep it warp-uniform) and one
+    // elected lane issues the copies: a single-lane loop issues bulk copies
+    // several times more slowly.
+    const bool leader = elect_one();
+    if (leader) {
+      mbar_arrive_expect_tx(xbar, (uint32_t)(p.M * p.d * 2));
+      for (int m = 0; m < p.M; ++m)
+        bulk_g2s(smem + xs_off + (size_t)m * xrow * 2, p.x + (size_t)(p.m0 + m) * p.d, (uint32_t)(p.d * 2), xbar);
+    }
     bool t_loaded = false;
     int it = 0;
     for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x) {
@@ -164,13 +169,17 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
         if (s == res_stages && !t_loaded) {
           // The rank-r fragments come from the pre-pass grid.
           asm volatile("griddepcontrol.wait;\n" ::: "memory");
-          mbar_arrive_expect_tx(tbar, (uint32_t)(p.nls * 1024));
-          bulk_g2s(smem + ts_off, p.ts, (uint32_t)(p.nls * 1024), tbar);
+          if (leader) {
+            mbar_arrive_expect_tx(tbar, (uint32_t)(p.nls * 1024));
+            bulk_g2s(smem + ts_off, p.ts, (uint32_t)(p.nls * 1024), tbar);
+          }
           t_loaded = true;
         }
-        if (!mbar_wait(&empty[st], ((it / stages) & 1) ^ 1, p.wait_budget, abort_flag, p.err)) goto producer_abort;
+        if (!mbar_wait_warp(&empty[st], ((it / stages) & 1) ^ 1, p.wait_budget, abort_flag, p.err))
+          goto producer_abort;
         uint8_t *buf = smem + (size_t)st * Geom::kBytes;
-        if (s < res_stages) {
+        if (!leader) {
+        } else if (s < res_stages) {
           const int kc0 = s * SC;
           const int g0 = (kc0 * kChunkK) / p.g;
           const int g1 = ((kc0 + SC) * kChunkK - 1) / p.g;
@@ -196,6 +205,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
                        &full[st]);
           }
         }
+        __syncwarp();
       }
     }
     return;
@@ -203,10 +213,10 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
     // Let copies already issued land before the block exits.
     for (int k = 1; k <= stages && it - k >= 0; ++k) {
       const int j = it - k;
-      mbar_wait(&full[j % stages], (j / stages) & 1, p.wait_budget, nullptr, p.err);
+      mbar_wait_warp(&full[j % stages], (j / stages) & 1, p.wait_budget, nullptr, p.err);
     }
-    mbar_wait(xbar, 0, p.wait_budget, nullptr, p.err);
-    if (t_loaded) mbar_wait(tbar, 0, p.wait_budget, nullptr, p.err);
+    mbar_wait_warp(xbar, 0, p.wait_budget, nullptr, p.err);
+    if (t_loaded) mbar_wait_warp(tbar, 0, p.wait_budget, nullptr, p.err);
     return;
   }
 
