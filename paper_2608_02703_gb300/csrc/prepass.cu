@@ -116,8 +116,20 @@ __global__ void __launch_bounds__(256) prepass_kernel(PrepassParams p) {
     // Tokens past M in this 16-token chunk get zero fragments.
     if (m >= mt && !p.ts) continue;
     float t = 0.f;
-    for (int sp = 0; sp < nsplit && m < mt; ++sp)
-      t += __ldcg(p.partial + ((int64_t)sp * gridDim.y * gridDim.x + pair) * (kPreTok * kPreCols) + e);
+    if (m < mt) {
+      // Eight loads in flight, added in split order.
+      const float *src = p.partial + (int64_t)pair * (kPreTok * kPreCols) + e;
+      const int64_t step = (int64_t)gridDim.y * gridDim.x * (kPreTok * kPreCols);
+      int sp = 0;
+      for (; sp + 8 <= nsplit; sp += 8) {
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[u] = __ldcg(src + (sp + u) * step);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) t += v[u];
+      }
+      for (; sp < nsplit; ++sp) t += __ldcg(src + sp * step);
+    }
     const int kk = c0 + c;
     if (kk < p.rcp) {
       t = kk < p.rc ? t * fp16_bits_to_f32(p.s_v[kk]) * fp16_bits_to_f32(p.s_u[kk]) : 0.f;
