@@ -5,13 +5,16 @@
 // Persistent grid, one block per SM.  A unit of work is 512 vocabulary rows
 // (four 128-row tiles).  One producer warp streams each unit's INT4 codes,
 // group scales and low-rank codes with 1-D bulk TMA copies into a ring of
-// shared-memory stages (mbarrier full/empty pairs).  Sixteen consumer warps each
-// own two 16-row m-tiles.  Per 16-wide k step a consumer turns one 32-bit
-// word of offset-binary nibbles into the four bf16 A-fragment registers of an
-// m16n8k16 MMA (exact small integers) and multiplies them with the bf16 hidden
-// states (B fragments, tokens on the 8-wide side, staged once per block by
-// TMA), accumulating in fp32.  At the end of every quantisation group the
-// partial sums are promoted by that row's group scale in fp32.  The rank-r
+// shared-memory stages (mbarrier full/empty pairs).  Eight consumer warps each
+// own four 16-row m-tiles.  The hidden states are staged once per block by
+// TMA and converted in place to fp16, each token scaled by a power of two that
+// keeps it in fp16 range (exact for bf16 inputs in the normal range).  Per
+// 16-wide k step a consumer turns one 32-bit word of offset-binary nibbles
+// into the four fp16 A-fragment registers of an m16n8k16 MMA (exact biased
+// integers, see unpack_int4x8_f16) and multiplies them with the hidden states
+// (B fragments, tokens on the 8-wide side), accumulating in fp32.  At the end
+// of every quantisation group the bias is removed and the partial sums are
+// promoted by that row's group scale in fp32.  The rank-r
 // branches follow as extra k steps: int8 codes of A_c (core) or A_w
 // (correction) times the bf16 hi/lo split of t = x V from the pre-pass, the
 // correction promoted by the row scale of A_w.  The pre-pass runs as the
@@ -58,7 +61,7 @@ static DecodePlan decode_plan(int d_pad, int nls, int g, int M) {
   const size_t stage_bytes = pl.sc == 2 ? StageGeom<2>::kBytes : StageGeom<1>::kBytes;
   const size_t xs_bytes = (size_t)M * xs_row_elems(d_pad) * 2;
   const size_t ts_bytes = (size_t)nls * 1024;
-  const size_t xsum_bytes = (size_t)(d_pad / g) * kDecodeMaxTokens * 4;
+  const size_t xsum_bytes = ((size_t)2 * (d_pad / g) * kDecodeMaxTokens + kDecodeMaxTokens) * 4;
   const size_t fixed = xs_bytes + ts_bytes + xsum_bytes + 256;
   const size_t shared_cap = (size_t)kSmemLimit - prepass_smem(M) - 2048;
   int st = 8;
@@ -77,18 +80,18 @@ static DecodePlan decode_plan(int d_pad, int nls, int g, int M) {
 }
 
 // Residual group promotion with the operand bias removed:
-// acc += s_row * (part + nb_tok), nb = -136 * sum of x over the group; part = 0.
-// Residual group promotion with the operand bias removed:
-// acc += s_row * (part + nb_tok), nb = -136 * sum of x over the group.
+// acc += s_row * (part + nb_tok), nb = -(operand bias) * sum of x over the
+// group, separately for rows gq (bias 1032) and gq + 8 (bias 1152; s_hi
+// carries the 1/16 of those rows' operands).
 template <int NT>
 __device__ __forceinline__ void promote_res(float (&acc)[NT][4], const float (&part)[NT][4], float s_lo, float s_hi,
-                                            const float2 (&nb)[NT]) {
+                                            const float2 (&nb_lo)[NT], const float2 (&nb_hi)[NT]) {
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) {
-    acc[nt][0] = fmaf(s_lo, part[nt][0] + nb[nt].x, acc[nt][0]);
-    acc[nt][1] = fmaf(s_lo, part[nt][1] + nb[nt].y, acc[nt][1]);
-    acc[nt][2] = fmaf(s_hi, part[nt][2] + nb[nt].x, acc[nt][2]);
-    acc[nt][3] = fmaf(s_hi, part[nt][3] + nb[nt].y, acc[nt][3]);
+    acc[nt][0] = fmaf(s_lo, part[nt][0] + nb_lo[nt].x, acc[nt][0]);
+    acc[nt][1] = fmaf(s_lo, part[nt][1] + nb_lo[nt].y, acc[nt][1]);
+    acc[nt][2] = fmaf(s_hi, part[nt][2] + nb_hi[nt].x, acc[nt][2]);
+    acc[nt][3] = fmaf(s_hi, part[nt][3] + nb_hi[nt].y, acc[nt][3]);
   }
 }
 
@@ -111,9 +114,11 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
   using Geom = StageGeom<SC>;
   constexpr int SS = 4 * SC;  // 16-wide k steps per stage
   extern __shared__ __align__(1024) uint8_t smem[];
-  const uint16_t *xs_s = reinterpret_cast<const uint16_t *>(smem + xs_off);
+  uint16_t *xs_s = reinterpret_cast<uint16_t *>(smem + xs_off);
   const uint32_t *ts_s = reinterpret_cast<const uint32_t *>(smem + ts_off);
-  float *xsum_s = reinterpret_cast<float *>(smem + xsum_off);  // [group][16 tokens]: -136 * sum of x
+  // [group][16 tokens] -1032 * sum of x, then the same with -1152, then the
+  // 16 tokens' scale factors (powers of two) that undo the fp16 staging scale.
+  float *xsum_s = reinterpret_cast<float *>(smem + xsum_off);
   uint64_t *full = reinterpret_cast<uint64_t *>(smem + bar_off);
   uint64_t *empty = full + 8;
   uint64_t *xbar = full + 16;
@@ -224,28 +229,56 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
   const int tsel = warp / (8 / kDecMT);              // tile of the unit
   const int mi0 = (warp % (8 / kDecMT)) * kDecMT;    // first of the warp's m-tiles in that tile
   const int gq = lane >> 2, cq = lane & 3;
+  const int ng = p.d_pad / p.g;
+  float *tscale = xsum_s + 2 * ng * kDecodeMaxTokens;
   {
-    // Per-group sums of the hidden states, for removing the operand bias.
     const bool ok = mbar_wait(xbar, 0, p.wait_budget, abort_flag, p.err);
-    const int ng = p.d_pad / p.g;
     if (ok) {
+      // Per-token power of two 2^-e that brings max |x| into [2^14, 2^15)
+      // (fp16 range, and small tokens away from fp16 subnormals); tscale[m]
+      // = 2^e undoes it after the residual.
+      for (int m = warp; m < kDecodeMaxTokens; m += kDecWarps) {
+        uint32_t mx = 0;
+        if (m < p.M) {
+          const uint32_t *row = reinterpret_cast<const uint32_t *>(xs_s + m * xrow);
+          for (int k = lane; k < p.d_pad / 2; k += 32) {
+            const uint32_t v = row[k];
+            mx = max(mx, max(v & 0x7FFFu, (v >> 16) & 0x7FFFu));
+          }
+        }
+        mx = __reduce_max_sync(0xffffffffu, mx);
+        const int ex = (int)(mx >> 7);             // biased bf16 exponent of the largest |x|
+        const int e = max(ex - 141, -126);       // max |x| < 2^(ex-126); 2^-e of it lies below 2^15
+        if (lane == 0) tscale[m] = __uint_as_float((uint32_t)(127 + e) << 23);
+      }
+      asm volatile("bar.sync 1, %0;\n" ::"r"(kDecWarps * 32) : "memory");
+      // Convert each token's row to fp16 in place, group by group, and sum
+      // the values the MMAs will see (for removing the operand bias).
       for (int e = threadIdx.x; e < ng * kDecodeMaxTokens; e += kDecWarps * 32) {
         const int grp = e / kDecodeMaxTokens, m = e % kDecodeMaxTokens;
         float sum = 0.f;
         if (m < p.M) {
-          const uint32_t *row = reinterpret_cast<const uint32_t *>(xs_s + m * xrow + grp * p.g);
+          const float inv = 1.f / tscale[m];  // exact: a power of two
+          uint32_t *row = reinterpret_cast<uint32_t *>(xs_s + m * xrow + grp * p.g);
           for (int k = 0; k < p.g / 2; ++k) {
             const uint32_t v = row[k];
-            sum += bf16_lo(v);
-            sum += bf16_hi(v);
+            const __half2 h = __floats2half2_rn(bf16_lo(v) * inv, bf16_hi(v) * inv);
+            row[k] = *reinterpret_cast<const uint32_t *>(&h);
+            sum += __low2float(h);
+            sum += __high2float(h);
           }
         }
-        xsum_s[e] = -kInt4Bias * sum;
+        xsum_s[e] = -kF16BiasLo * sum;
+        xsum_s[ng * kDecodeMaxTokens + e] = -kF16BiasHi * sum;
       }
     }
     asm volatile("bar.sync 1, %0;\n" ::"r"(kDecWarps * 32) : "memory");  // consumer warps only
     if (!ok) return;
   }
+  // Factors that undo the staging scale for this lane's two token columns.
+  float2 unscale[NT];
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) unscale[nt] = make_float2(tscale[8 * nt + 2 * cq], tscale[8 * nt + 2 * cq + 1]);
   // B-fragment bases: token 8*nt + gq (clamped to the M rows held; the extra
   // columns are never stored), column 2*cq (+ 16 per k step, + 8 for b1).
   const uint16_t *xb[NT];
@@ -289,7 +322,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
 #pragma unroll
           for (int mt = 0; mt < kDecMT; ++mt) {
             s_lo[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16]);
-            s_hi[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16 + 8]);
+            s_hi[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16 + 8]) * 0.0625f;  // operands x16
           }
       }
       __syncwarp();
@@ -313,15 +346,15 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
           for (int mt = 0; mt < kDecMT; ++mt) {
             const uint32_t word = j == 0 ? w[c][mt].x : j == 1 ? w[c][mt].y : j == 2 ? w[c][mt].z : w[c][mt].w;
             uint32_t a[4];
-            unpack_int4x8_biased(word, a);
+            unpack_int4x8_f16(word, a);
             // First k step of a group: compile-time when groups fit in a stage.
             const bool first = GS <= SS ? (ks % GS == 0) : (ks == 0 && (s % (GS / SS)) == 0);
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
               if (first)
-                mma_bf16_16816_zero(part[mt][nt], a, b[nt][0], b[nt][1]);
+                mma_f16_16816_zero(part[mt][nt], a, b[nt][0], b[nt][1]);
               else
-                mma_bf16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
+                mma_f16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
             }
           }
           // Group boundary: compile-time inside a stage when GS <= SS; every
@@ -330,16 +363,31 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
           if (boundary) {
             const int gi = GS <= SS ? ks / GS : 0;                               // group within the stage
             const int ggl = GS <= SS ? s * (SS / GS) + ks / GS : s / (GS / SS);  // group index along d
-            float2 nb[NT];
+            float2 nb_lo[NT], nb_hi[NT];
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt)
-              nb[nt] = *reinterpret_cast<const float2 *>(xsum_s + ggl * kDecodeMaxTokens + 8 * nt + 2 * cq);
+            for (int nt = 0; nt < NT; ++nt) {
+              const int o = ggl * kDecodeMaxTokens + 8 * nt + 2 * cq;
+              nb_lo[nt] = *reinterpret_cast<const float2 *>(xsum_s + o);
+              nb_hi[nt] = *reinterpret_cast<const float2 *>(xsum_s + ng * kDecodeMaxTokens + o);
+            }
 #pragma unroll
-            for (int mt = 0; mt < kDecMT; ++mt) promote_res<NT>(acc[mt], part[mt], s_lo[gi][mt], s_hi[gi][mt], nb);
+            for (int mt = 0; mt < kDecMT; ++mt)
+              promote_res<NT>(acc[mt], part[mt], s_lo[gi][mt], s_hi[gi][mt], nb_lo, nb_hi);
           }
         }
       }
     }
+
+    // Back to the hidden states' own scale (exact: powers of two).
+#pragma unroll
+    for (int a = 0; a < kDecMT; ++a)
+#pragma unroll
+      for (int b = 0; b < NT; ++b) {
+        acc[a][b][0] *= unscale[b].x;
+        acc[a][b][1] *= unscale[b].y;
+        acc[a][b][2] *= unscale[b].x;
+        acc[a][b][3] *= unscale[b].y;
+      }
 
     // Rank-r branches as extra k steps (core: factor 1; correction: row scale
     // of A_w), with the same copy-then-release of each stage.

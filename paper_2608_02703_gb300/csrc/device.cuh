@@ -48,6 +48,25 @@ __device__ __forceinline__ void unpack_int4x8_biased(uint32_t w, uint32_t (&a)[4
 
 constexpr float kInt4Bias = 136.0f;
 
+// fp16 operands for the decode kernel: OR-ing a nibble into the mantissa of
+// fp16 1024.0 is exact at bits 0-3 (1024 + n) and at bits 4-7 (1024 + 16 n),
+// so a word's eight nibbles need one shift and four LOP3s.  Registers a[0],
+// a[2] (rows gq of the m16n8k16 A fragment) hold 1024 + n = 1032 + code;
+// a[1], a[3] (rows gq + 8) hold 1024 + 16 n = 1152 + 16 code.  The kernel
+// removes 1032 * sum(x) resp. 1152 * sum(x) per group and scales rows gq + 8
+// by 1/16 at promotion.
+constexpr float kF16BiasLo = 1032.0f;
+constexpr float kF16BiasHi = 1152.0f;
+
+__device__ __forceinline__ void unpack_int4x8_f16(uint32_t w, uint32_t (&a)[4]) {
+  const uint32_t kMagic = 0x64006400u;  // fp16 1024.0 | 1024.0
+  const uint32_t t = w >> 8;
+  a[0] = lop3_and_or(w, 0x000F000Fu, kMagic);
+  a[1] = lop3_and_or(w, 0x00F000F0u, kMagic);
+  a[2] = lop3_and_or(t, 0x000F000Fu, kMagic);
+  a[3] = lop3_and_or(t, 0x00F000F0u, kMagic);
+}
+
 // Exact codes: the biased operands minus 136.0 (exact in bf16).
 __device__ __forceinline__ void unpack_int4x8(uint32_t w, uint32_t (&a)[4]) {
   constexpr uint32_t kBias = 0x43084308u;  // bf16 136.0 | 136.0
@@ -100,6 +119,23 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a
 __device__ __forceinline__ void mma_bf16_16816_zero(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
   asm volatile(
       "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%10,%10,%10};\n"
+      : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(0.f));
+}
+
+// fp16 x fp16 -> fp32 variants (the decode kernel's residual operands).
+__device__ __forceinline__ void mma_f16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ void mma_f16_16816_zero(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
       "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%10,%10,%10};\n"
       : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(0.f));

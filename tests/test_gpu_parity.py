@@ -84,6 +84,26 @@ def test_decode_logits(name, M):
     gu.check_logits(got16, ref, bf16=True, where=f"{name} M={M} bf16")
 
 
+@pytest.mark.parametrize("M", [1, 2, 12])
+def test_decode_hidden_state_range(M):
+    """Hidden states far outside fp16 range, or tiny, one scale per token: the
+    decode path stages them in fp16 under a per-token power-of-two scale."""
+    pack, head = get("tiny")
+    shape = SHAPES["tiny"]
+    x = make_hidden(shape.d, M, seed=50 + M).view(np.uint16).astype(np.uint32)
+    # Shift bf16 exponents by +14 or -40 (powers of two: exact), alternating per token.
+    shift = np.where(np.arange(M) % 2 == 0, 14, -40)[:, None].astype(np.int64)
+    exp = ((x >> 7) & 0xFF).astype(np.int64)
+    nz = exp > 0
+    new_exp = np.where(nz, exp + shift, 0)
+    assert new_exp.max() < 255 and new_exp[nz].min() > 0
+    xs = ((x & 0x807F) | (new_exp.astype(np.uint32) << 7)).astype(np.uint16)
+    ref = oracle.logits(head, shape, xs)
+    got = gu.forward(pack, xs, archead.OUT_FP32, archead.PATH_DECODE)
+    for m in range(M):  # each token against its own scale
+        gu.check_logits(got[m:m + 1], ref[m:m + 1], where=f"M={M} token {m}")
+
+
 @pytest.mark.parametrize("name", ["ragged", "tiny", "g32", "max_rank"])
 @pytest.mark.parametrize("M", [17, 40, 133])
 def test_logits_many_tokens(name, M):
