@@ -183,7 +183,9 @@ ARCHEAD_API archead_status archead_debug_dequant(const archead_pack *pack, int c
 
 /*
  * Wait for the stream, then read and clear the pack's device error word.
- * Returns ARCHEAD_OK, ARCHEAD_ERR_TARGET_RANGE, ARCHEAD_ERR_DEVICE_TIMEOUT or
+ * Returns ARCHEAD_OK, ARCHEAD_ERR_TARGET_RANGE, ARCHEAD_ERR_DEVICE_TIMEOUT,
+ * ARCHEAD_ERR_UNSUPPORTED (a kernel found its shared-memory window misaligned
+ * for its TMA layout and skipped its work; archead_last_error() says so) or
  * ARCHEAD_ERR_CUDA.
  */
 ARCHEAD_API archead_status archead_sync_status(archead_pack *pack, void *stream);

@@ -495,6 +495,10 @@ archead_status archead_sync_status(archead_pack *pack, void *stream) {
   AH_CUDA(cudaMemset(pack->err, 0, sizeof(int)));
   if (word & kErrWaitTimeout) return ARCHEAD_ERR_DEVICE_TIMEOUT;
   if (word & kErrTargetRange) return ARCHEAD_ERR_TARGET_RANGE;
+  if (word & kErrLayout) {
+    set_last_error_message("a kernel found its shared-memory window misaligned for its TMA layout and skipped its work");
+    return ARCHEAD_ERR_UNSUPPORTED;
+  }
   return ARCHEAD_OK;
 }
 

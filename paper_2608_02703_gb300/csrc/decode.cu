@@ -35,12 +35,21 @@ constexpr int kSmemLimit = 227 * 1024;
 // shared-memory plan and the kernel instance launched both take it from here.
 __host__ __device__ constexpr int stage_chunks(int NT) { return NT == 1 ? 2 : 1; }
 
+// Instances with two n-tiles (9..16 tokens) do not keep the hidden states in
+// shared memory (16 rows of d would take most of it, leaving too shallow a
+// ring to stream at full bandwidth).  Each residual stage instead carries the
+// matching 64-wide chunks of x for 16 tokens, loaded by a 2-D TMA copy, and
+// those instances multiply bf16 operands (no fp16 staging).
+__host__ __device__ constexpr bool streams_x(int NT) { return NT == 2; }
+constexpr int kXChunkBytes = 16 * kChunkK * 2;  // 16 tokens x 64 of d, bf16, 128-byte swizzle
+
 // Stage geometry for SC chunks (64 of d each) per stage.
-template <int SC>
+template <int SC, bool XS>
 struct StageGeom {
   static constexpr int kCodeBytes = kDecTiles * SC * kChunkBytes;  // also holds 2*SC low-rank steps per tile
   static constexpr int kScaleBytesPerTile = (SC * kChunkK / 32) * kTileRows * 2;  // up to SC*64/g groups (g >= 32)
-  static constexpr int kBytes = kCodeBytes + kDecTiles * kScaleBytesPerTile;
+  static constexpr int kXOff = kCodeBytes + kDecTiles * kScaleBytesPerTile;       // a multiple of 1024
+  static constexpr int kBytes = kXOff + (XS ? SC * kXChunkBytes : 0);
   static constexpr int kLrSteps = 2 * SC;  // 16-wide low-rank steps per stage (2 KB per tile each)
 };
 
@@ -57,9 +66,12 @@ __host__ __device__ __forceinline__ int xs_row_elems(int d_pad) { return d_pad +
 // overlaps the two grids) whenever the stage ring still holds 96 KB.
 static DecodePlan decode_plan(int d_pad, int nls, int g, int M) {
   DecodePlan pl{};
-  pl.sc = stage_chunks(M > 8 ? 2 : 1);
-  const size_t stage_bytes = pl.sc == 2 ? StageGeom<2>::kBytes : StageGeom<1>::kBytes;
-  const size_t xs_bytes = (size_t)M * xs_row_elems(d_pad) * 2;
+  const int nt = M > 8 ? 2 : 1;
+  const bool xs = streams_x(nt);
+  pl.sc = stage_chunks(nt);
+  const size_t stage_bytes = pl.sc == 2 ? (xs ? StageGeom<2, true>::kBytes : StageGeom<2, false>::kBytes)
+                                        : (xs ? StageGeom<1, true>::kBytes : StageGeom<1, false>::kBytes);
+  const size_t xs_bytes = xs ? 0 : (size_t)M * xs_row_elems(d_pad) * 2;
   const size_t ts_bytes = (size_t)nls * 1024;
   const size_t xsum_bytes = ((size_t)2 * (d_pad / g) * kDecodeMaxTokens + kDecodeMaxTokens) * 4;
   const size_t fixed = xs_bytes + ts_bytes + xsum_bytes + 256;
@@ -109,11 +121,21 @@ __device__ __forceinline__ void promote(float (&acc)[NT][4], const float (&part)
 
 // NT: n-tiles of 8 tokens; SC: 64-wide chunks per stage; GS: 16-wide k steps per group.
 template <int NT, int SC, int GS>
-__global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, int stages, int xs_off, int ts_off,
-                                                                int xsum_off, int bar_off) {
-  using Geom = StageGeom<SC>;
+__global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_constant__ DecodeParams p, int stages,
+                                                                int xs_off, int ts_off, int xsum_off, int bar_off) {
+  constexpr bool kStreamX = streams_x(NT);
+  constexpr bool kF16 = !kStreamX;  // fp16 operands with x staged in shared memory
+  using Geom = StageGeom<SC, kStreamX>;
   constexpr int SS = 4 * SC;  // 16-wide k steps per stage
+  // The kernel has no static shared memory, so the dynamic window starts on a
+  // 1 KB boundary, which the 128-byte-swizzled x boxes rely on (checked
+  // below).  Offsets from this base stay compile-time friendly; a rounded-up
+  // runtime base made the inner loops measurably slower.
   extern __shared__ __align__(1024) uint8_t smem[];
+  if (kStreamX && (smem_u32(smem) & 1023u) != 0) {
+    if (threadIdx.x == 0) atomicOr(p.err, kErrLayout);
+    return;
+  }
   uint16_t *xs_s = reinterpret_cast<uint16_t *>(smem + xs_off);
   const uint32_t *ts_s = reinterpret_cast<const uint32_t *>(smem + ts_off);
   // [group][16 tokens] -1032 * sum of x, then the same with -1152, then the
@@ -135,7 +157,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
 
   // Columns [d, d_pad) of the hidden states meet zero codes; zero them so
   // that no stale pattern (a NaN) reaches the accumulators.
-  if (p.d < p.d_pad) {
+  if (!kStreamX && p.d < p.d_pad) {
     const int per_row = (p.d_pad - p.d) / 8;  // uint4 per row
     for (int e = threadIdx.x; e < p.M * per_row; e += blockDim.x) {
       uint4 *dst = reinterpret_cast<uint4 *>(smem + xs_off + (size_t)(e / per_row) * xrow * 2 + (size_t)p.d * 2);
@@ -160,7 +182,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
     // elected lane issues the copies: a single-lane loop issues bulk copies
     // several times more slowly.
     const bool leader = elect_one();
-    if (leader) {
+    if (!kStreamX && leader) {
       mbar_arrive_expect_tx(xbar, (uint32_t)(p.M * p.d * 2));
       for (int m = 0; m < p.M; ++m)
         bulk_g2s(smem + xs_off + (size_t)m * xrow * 2, p.x + (size_t)(p.m0 + m) * p.d, (uint32_t)(p.d * 2), xbar);
@@ -189,7 +211,12 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
           const int g0 = (kc0 * kChunkK) / p.g;
           const int g1 = ((kc0 + SC) * kChunkK - 1) / p.g;
           const int ng = g1 - g0 + 1;
-          mbar_arrive_expect_tx(&full[st], (uint32_t)(ntile * (SC * kChunkBytes + ng * kTileRows * 2)));
+          mbar_arrive_expect_tx(&full[st],
+                                (uint32_t)(ntile * (SC * kChunkBytes + ng * kTileRows * 2) + (kStreamX ? SC * kXChunkBytes : 0)));
+          if (kStreamX) {
+            for (int c = 0; c < SC; ++c)
+              tma_load_2d(buf + Geom::kXOff + c * kXChunkBytes, &p.tmap_x, (kc0 + c) * kChunkK, p.m0, &full[st]);
+          }
           for (int t = 0; t < ntile; ++t) {
             const int64_t vt = (int64_t)kDecTiles * unit + t;
             bulk_g2s(buf + t * SC * kChunkBytes, p.codes + (vt * KC + kc0) * kChunkBytes, SC * kChunkBytes, &full[st]);
@@ -220,7 +247,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
       const int j = it - k;
       mbar_wait_warp(&full[j % stages], (j / stages) & 1, p.wait_budget, nullptr, p.err);
     }
-    mbar_wait_warp(xbar, 0, p.wait_budget, nullptr, p.err);
+    if (!kStreamX) mbar_wait_warp(xbar, 0, p.wait_budget, nullptr, p.err);
     if (t_loaded) mbar_wait_warp(tbar, 0, p.wait_budget, nullptr, p.err);
     return;
   }
@@ -231,7 +258,26 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
   const int gq = lane >> 2, cq = lane & 3;
   const int ng = p.d_pad / p.g;
   float *tscale = xsum_s + 2 * ng * kDecodeMaxTokens;
-  {
+  if (kStreamX) {
+    // Per-group sums of x for removing the bf16 operand bias (136), read
+    // straight from global memory; no staging scale.
+    for (int e = threadIdx.x; e < ng * kDecodeMaxTokens; e += kDecWarps * 32) {
+      const int grp = e / kDecodeMaxTokens, m = e % kDecodeMaxTokens;
+      float sum = 0.f;
+      if (m < p.M && grp * p.g < p.d) {
+        const uint4 *src = reinterpret_cast<const uint4 *>(p.x + (int64_t)(p.m0 + m) * p.d + (int64_t)grp * p.g);
+        for (int q = 0; q < p.g / 8; ++q) {
+          const uint4 v = src[q];
+          sum += bf16_lo(v.x) + bf16_hi(v.x) + bf16_lo(v.y) + bf16_hi(v.y);
+          sum += bf16_lo(v.z) + bf16_hi(v.z) + bf16_lo(v.w) + bf16_hi(v.w);
+        }
+      }
+      xsum_s[e] = -kInt4Bias * sum;
+      xsum_s[ng * kDecodeMaxTokens + e] = -kInt4Bias * sum;
+    }
+    if (threadIdx.x < kDecodeMaxTokens) tscale[threadIdx.x] = 1.f;
+    asm volatile("bar.sync 1, %0;\n" ::"r"(kDecWarps * 32) : "memory");  // consumer warps only
+  } else {
     const bool ok = mbar_wait(xbar, 0, p.wait_budget, abort_flag, p.err);
     if (ok) {
       // Per-token power of two 2^-e that brings max |x| into [2^14, 2^15)
@@ -283,7 +329,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
   // columns are never stored), column 2*cq (+ 16 per k step, + 8 for b1).
   const uint16_t *xb[NT];
 #pragma unroll
-  for (int nt = 0; nt < NT; ++nt) xb[nt] = xs_s + min(8 * nt + gq, p.M - 1) * xrow + 2 * cq;
+  for (int nt = 0; nt < NT; ++nt) xb[nt] = kStreamX ? nullptr : xs_s + min(8 * nt + gq, p.M - 1) * xrow + 2 * cq;
   bool t_ready = false;
 
   int st = 0;     // ring slot
@@ -308,6 +354,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
       if (!mbar_wait(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
       uint4 w[SC][kDecMT];
       float s_lo[NGS][kDecMT], s_hi[NGS][kDecMT];
+      uint32_t bx[kStreamX ? SS : 1][NT][2];  // streamed x: this stage's B fragments
       if (active) {
         const uint8_t *buf = smem + (size_t)st * Geom::kBytes;
         const uint8_t *cb = buf + tsel * SC * kChunkBytes + mi0 * 512 + lane * 16;
@@ -322,8 +369,21 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
 #pragma unroll
           for (int mt = 0; mt < kDecMT; ++mt) {
             s_lo[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16]);
-            s_hi[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16 + 8]) * 0.0625f;  // operands x16
+            s_hi[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16 + 8]) * (kF16 ? 0.0625f : 1.f);  // fp16: x16
           }
+        if (kStreamX) {
+          // Token 8*nt + gq, k = 16*ks + 2*cq (+8): 128-byte rows, 16-byte
+          // chunk index XOR (row % 8) = gq.
+#pragma unroll
+          for (int ks = 0; ks < (kStreamX ? SS : 1); ++ks)
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+              const uint8_t *xr = buf + Geom::kXOff + (ks >> 2) * kXChunkBytes + (8 * nt + gq) * 128 + 4 * cq;
+              const int ch = 2 * (ks & 3);
+              bx[ks][nt][0] = *reinterpret_cast<const uint32_t *>(xr + ((ch ^ gq) << 4));
+              bx[ks][nt][1] = *reinterpret_cast<const uint32_t *>(xr + (((ch + 1) ^ gq) << 4));
+            }
+        }
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty[st]);
@@ -338,23 +398,38 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
           uint32_t b[NT][2];
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
-            const uint16_t *q = xb[nt] + kbase + ks * 16;
-            b[nt][0] = *reinterpret_cast<const uint32_t *>(q);
-            b[nt][1] = *reinterpret_cast<const uint32_t *>(q + 8);
+            if (kStreamX) {
+              b[nt][0] = bx[kStreamX ? ks : 0][nt][0];
+              b[nt][1] = bx[kStreamX ? ks : 0][nt][1];
+            } else {
+              const uint16_t *q = xb[nt] + kbase + ks * 16;
+              b[nt][0] = *reinterpret_cast<const uint32_t *>(q);
+              b[nt][1] = *reinterpret_cast<const uint32_t *>(q + 8);
+            }
           }
 #pragma unroll
           for (int mt = 0; mt < kDecMT; ++mt) {
             const uint32_t word = j == 0 ? w[c][mt].x : j == 1 ? w[c][mt].y : j == 2 ? w[c][mt].z : w[c][mt].w;
             uint32_t a[4];
-            unpack_int4x8_f16(word, a);
+            if (kF16)
+              unpack_int4x8_f16(word, a);
+            else
+              unpack_int4x8_biased(word, a);
             // First k step of a group: compile-time when groups fit in a stage.
             const bool first = GS <= SS ? (ks % GS == 0) : (ks == 0 && (s % (GS / SS)) == 0);
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
-              if (first)
-                mma_f16_16816_zero(part[mt][nt], a, b[nt][0], b[nt][1]);
-              else
-                mma_f16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
+              if (kF16) {
+                if (first)
+                  mma_f16_16816_zero(part[mt][nt], a, b[nt][0], b[nt][1]);
+                else
+                  mma_f16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
+              } else {
+                if (first)
+                  mma_bf16_16816_zero(part[mt][nt], a, b[nt][0], b[nt][1]);
+                else
+                  mma_bf16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
+              }
             }
           }
           // Group boundary: compile-time inside a stage when GS <= SS; every
@@ -380,7 +455,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(DecodeParams p, 
 
     // Back to the hidden states' own scale (exact: powers of two).
 #pragma unroll
-    for (int a = 0; a < kDecMT; ++a)
+    for (int a = 0; a < (kF16 ? kDecMT : 0); ++a)
 #pragma unroll
       for (int b = 0; b < NT; ++b) {
         acc[a][b][0] *= unscale[b].x;
@@ -571,7 +646,10 @@ cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool
   static_assert(stage_chunks(1) >= 1 && stage_chunks(2) >= 1, "stage width");
   if ((dp.NT == 1) != (dp.M <= 8) || pl.sc != stage_chunks(dp.NT)) return cudaErrorInvalidValue;
   if (dp.NT == 1) return launch_g<1, stage_chunks(1)>(dp, grid, s, pl, pdl);
-  return launch_g<2, stage_chunks(2)>(dp, grid, s, pl, pdl);
+  static_assert(streams_x(2) && !streams_x(1), "two n-tiles stream x");
+  DecodeParams dx = dp;
+  if (!make_tma_map_bf16(&dx.tmap_x, dp.x, dp.M_total, dp.d, 16)) return cudaErrorInvalidValue;
+  return launch_g<2, stage_chunks(2)>(dx, grid, s, pl, pdl);
 }
 
 }  // namespace archead

@@ -12,6 +12,7 @@ namespace archead {
 // Bits of the per-pack device error word.
 constexpr int kErrWaitTimeout = 1;
 constexpr int kErrTargetRange = 2;
+constexpr int kErrLayout = 4;  // a kernel found its shared memory misaligned and did nothing
 
 // ---------------------------------------------------------------------------
 // INT4 / INT8 code unpacking to exact bf16 operands.
@@ -232,6 +233,17 @@ __device__ __forceinline__ bool mbar_wait_warp(uint64_t *bar, uint32_t parity, i
       return false;
     }
   }
+}
+
+// 2-D tensor copy (TMA) of one box at (c0 = column, c1 = row) into shared
+// memory, completing on an mbarrier.  c0 * element size must be a multiple
+// of 16 bytes.
+__device__ __forceinline__ void tma_load_2d(void *dst, const void *map, int c0, int c1, uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];\n" ::"r"(
+          smem_u32(dst)),
+      "l"(map), "r"(c0), "r"(c1), "r"(smem_u32(bar))
+      : "memory");
 }
 
 // Global -> shared bulk copy completing on an mbarrier (size multiple of 16,

@@ -26,6 +26,7 @@
 //  Correction row scales: [V_pad] fp16 bits (zero on padding rows).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -45,6 +46,7 @@ constexpr int kPrepassKSplit = 256;  // d per pre-pass block
 constexpr int64_t kDefaultWaitBudget = 2000000000LL;  // cycles, about one second
 
 struct DecodeParams {
+  CUtensorMap tmap_x;   // x [M_total][d] bf16, box 64 x 16 rows (kernel instances that stream x; M > 8)
   const uint8_t *codes;
   const uint16_t *scales;
   const uint8_t *lr_codes;
@@ -136,6 +138,11 @@ size_t prepass_smem(int M);  // dynamic shared memory of one pre-pass block
 size_t prepass_partial_bytes(int M, int lr, int d);
 // pdl: launch as a programmatic dependent of the immediately preceding pre-pass grid.
 cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool pdl);
+// Tensor map of a bf16 [rows][cols] row-major matrix: box 64 columns x
+// box_rows rows, 128-byte swizzle, zero fill out of bounds.  False if the
+// driver entry point is missing or the encoder rejects the layout (base or
+// row pitch not 16-byte aligned).
+bool make_tma_map_bf16(CUtensorMap *map, const void *base, int64_t rows, int64_t cols, int box_rows);
 int decode_num_units(const archead_pack *p);
 int decode_parts_per_unit();
 bool decode_supported(int d_pad, int nls, int g);

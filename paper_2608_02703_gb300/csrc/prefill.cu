@@ -56,14 +56,6 @@ struct PrefillParams {
 // ------------------------------------------------------------------------
 // tcgen05 / TMA wrappers (inline PTX).
 // ------------------------------------------------------------------------
-__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int c0, int c1, uint64_t *bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];\n" ::"r"(
-          smem_u32(dst)),
-      "l"(map), "r"(c0), "r"(c1), "r"(smem_u32(bar))
-      : "memory");
-}
-
 __device__ __forceinline__ void tmem_alloc(uint32_t *slot, uint32_t cols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(slot)), "r"(cols)
                : "memory");
@@ -474,44 +466,15 @@ done:
 // ------------------------------------------------------------------------
 // Host side: tensor maps and launch.
 // ------------------------------------------------------------------------
-typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
-                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-static EncodeTiledFn encode_fn() {
-  static EncodeTiledFn fn = nullptr;
-  if (!fn) {
-    void *ptr = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(ptr);
-  }
-  return fn;
-}
-
-// bf16 [rows][cols] row-major, box 64 columns x 128 rows, 128-byte swizzle, zero fill out of bounds.
-static bool make_map(CUtensorMap *map, const void *base, int64_t rows, int64_t cols) {
-  EncodeTiledFn fn = encode_fn();
-  if (!fn) return false;
-  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
-  cuuint32_t box[2] = {64, 128};
-  cuuint32_t elem[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, elem,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 int prefill_parts_per_vt() { return 4; }
 
 cudaError_t launch_prefill(const archead_pack *pk, const void *x, int M, const uint16_t *T, void *out, int out_fp32,
                            const int32_t *targets, float2 *ce_part, float *ce_tlogit, cudaStream_t s) {
   PrefillParams p{};
-  if (!make_map(&p.tmap_x, x, M, pk->d)) return cudaErrorInvalidValue;
+  if (!make_tma_map_bf16(&p.tmap_x, x, M, pk->d, 128)) return cudaErrorInvalidValue;
   const int kt = 2 * (pk->rcp + pk->rrp);
   if (kt > 0) {
-    if (!make_map(&p.tmap_t, T, M, kt)) return cudaErrorInvalidValue;
+    if (!make_tma_map_bf16(&p.tmap_t, T, M, kt, 128)) return cudaErrorInvalidValue;
   }
   p.codes = pk->codes;
   p.scales = pk->scales;
