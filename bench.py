@@ -47,6 +47,39 @@ WORKLOADS = {
 }
 
 
+KERNEL_SOURCES = {
+    "decode": ("decode.cu", "device.cuh", "internal.h"),
+    "prefill": ("prefill.cu", "device.cuh", "internal.h"),
+}
+
+
+def kernel_source_hash(kernel: str) -> str:
+    """sha256 over the sources a kernel is compiled from (its traffic figure
+    is only valid for the sources it was captured with)."""
+    import hashlib
+
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES[kernel]:
+        with open(os.path.join(ROOT, "paper_2608_02703_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def captured_traffic(kernel: str, workload: str, M: int):
+    """DRAM bytes (read + write) per launch of `kernel` from the committed ncu
+    capture summary (profiles/traffic.json), or None if there is none for this
+    workload or the kernel's sources changed since it was taken."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        table = json.load(f)
+    e = table.get(f"{kernel}/{workload}/M={M}")
+    if not e or e.get("sources_sha256") != kernel_source_hash(kernel):
+        return None
+    return e["dram_bytes_per_launch"]
+
+
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -297,14 +330,16 @@ def run_ours(args, rank, world, local_rank):
     if M <= 64:
         achieved = kb / (kms / 1e3) / 1e9
         roof = {"kernel": main_kernel, "bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"],
-                "unit": "GB/s", "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": None,
+                "unit": "GB/s", "frac": round(achieved / peaks["hbm_gbs"], 4),
+                "traffic": captured_traffic(main_kernel, args.workload, M),
                 "peak_source": peak_src, "algorithmic_bytes_per_launch": kb, "mean_launch_ms": kms}
     else:
         fl = call_flops(shape, M) / prof[main_kernel]["launches_per_step"]
         achieved = fl / (kms / 1e3) / 1e12
         peak = peaks["bf16_tflops"]
         roof = {"kernel": main_kernel, "bound": "tensor", "achieved": round(achieved, 1), "peak": peak,
-                "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "traffic": None, "peak_source": peak_src,
+                "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
+                "traffic": captured_traffic(main_kernel, args.workload, M), "peak_source": peak_src,
                 "algorithmic_flops_per_launch": fl, "mean_launch_ms": kms}
 
     # End to end through the public host-buffer entry point.
