@@ -104,7 +104,7 @@ cudaError_t ensure_counters(archead_pack *p, int n, cudaStream_t s) {
 }
 
 struct ForwardPlan {
-  size_t partial_off = 0, t_off = 0, ce_part_off = 0, tlogit_off = 0, total = 0;
+  size_t partial_off = 0, ts_off = 0, ce_part_off = 0, tlogit_off = 0, total = 0;
   int nchunks = 0;
 };
 
@@ -114,7 +114,7 @@ ForwardPlan plan_decode(archead_pack *p, int64_t M, bool ce) {
   Carve c;
   f.nchunks = (int)((M + kDecodeMaxTokens - 1) / kDecodeMaxTokens);
   f.partial_off = c.take(prepass_partial_bytes((int)M, p->lr, p->d));
-  f.t_off = c.take((size_t)M * std::max(2 * p->lr, 64) * 2);
+  f.ts_off = c.take((size_t)f.nchunks * std::max(p->nls, 1) * 1024);
   if (ce) {
     f.ce_part_off = c.take((size_t)decode_num_units(p) * decode_parts_per_unit() * M * sizeof(float2));
     f.tlogit_off = c.take((size_t)M * sizeof(float));
@@ -166,8 +166,8 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   PrepassParams pp = prepass_params(p, x, M);
   pp.partial = at<float>(p->ws, f.partial_off);
   pp.counters = p->counters;
-  pp.ts = nullptr;
-  pp.T = at<uint16_t>(p->ws, f.t_off);
+  pp.ts = at<uint32_t>(p->ws, f.ts_off);
+  pp.T = nullptr;
   AH_CUDA(launch_prepass(pp, s, p));
 
   DecodeParams dp{};
@@ -184,8 +184,6 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   dp.g = p->g;
   dp.nls = p->nls;
   dp.nls_core = p->nls_core;
-  dp.rcp = p->rcp;
-  dp.rrp = p->rrp;
   dp.out = out;
   dp.out_fp32 = out_fp32;
   dp.targets = targets;
@@ -198,11 +196,13 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   for (int c = 0; c < f.nchunks; ++c) {
     dp.m0 = c * kDecodeMaxTokens;
     dp.M = (int)std::min<int64_t>(kDecodeMaxTokens, M - dp.m0);
+    dp.NT = dp.M > 8 ? 2 : 1;
+    dp.ts = pp.ts + (size_t)c * p->nls * 256;
     cudaEvent_t ev = nullptr;
     timer_begin(p, "decode", s, &ev);
     // The first chunk overlaps the pre-pass grid (programmatic dependent launch).
     const bool pdl = c == 0 && p->lr > 0 && !p->profiling;
-    cudaError_t e = launch_decode(dp, pp.T, grid, s, pdl);
+    cudaError_t e = launch_decode(dp, grid, s, pdl);
     timer_end(p, "decode", s, ev);
     if (e != cudaSuccess) return cuda_status(e);
   }

@@ -2,17 +2,15 @@
 //
 // Device layouts (all built by archead_pack_create from the canonical layout):
 //
-//  Residual codes, row-major tiles.  The vocabulary is cut into tiles of 128
-//  rows (V padded with zero rows), d (padded with zero codes to D_PAD, a
-//  multiple of 128) into chunks of 64.  Chunk (vt, kc) is 4 KB: [row 0..127]
-//  [32 bytes] = eight 32-bit words per row; word q of a row holds its 8 codes
-//  for columns 64*kc + 8q .. +7: nibble p (bits 4p..4p+3) is column 8q + 2p
-//  for p < 4 and 8q + 2(p-4) + 1 for p >= 4, so nibbles p and p+4 form the
-//  consecutive pair (8q+2p, 8q+2p+1).  Codes are stored offset-binary
-//  (code + 8).  A thread that owns a row turns its 32 bytes into 32 packed
-//  pairs in column order (one tensor-memory column or 4 bytes of a K-major
-//  shared-memory row each).
-//    byte offset = ((vt*KC + kc)*128 + row)*32 + 4q,   KC = D_PAD/64
+//  Residual codes, "fragment-native" tiling.  The vocabulary is cut into
+//  tiles of 128 rows (V padded with zero rows), d (padded with zero codes to
+//  D_PAD, a multiple of 128) into chunks of 64.  Chunk
+//  (vt, kc) is 4 KB: [mi 0..7][lane 0..31][word j 0..3] of 32-bit words.
+//  Word j of lane (gq = lane/4, cq = lane%4) in m-tile mi holds the 8 codes an
+//  m16n8k16 A-fragment needs for k16-step 4*kc + j: nibble p (pair i = p%4,
+//  half h = p/4) is row 16*mi + gq + 8*(i%2), column 16*(4*kc+j) + 2*cq +
+//  8*(i/2) + h.  Codes are stored offset-binary (code + 8).
+//    byte offset = ((((vt*KC + kc)*8 + mi)*32 + lane)*4 + j)*4,   KC = D_PAD/64
 //
 //  Residual scales: [vt][G_PAD][128] fp16 bits (row within tile fastest),
 //  G_PAD = D_PAD/g; scales of padding groups and rows are zero.
@@ -20,9 +18,10 @@
 //  Low-rank codes: the extended rank axis kk in [0, LR) with LR = RCP + RRP,
 //  RCP = r_c rounded up to 32, RRP = r_r rounded up to 32: kk < RCP is
 //  core_u[:, kk], kk >= RCP is corr_a[:, kk - RCP] (zero beyond the rank).
-//  Step ls (16 wide) of tile vt is 2 KB: [row 0..127][16 bytes], byte j =
-//  column 16*ls + j, stored offset-binary (code + 128).
-//    byte offset = ((vt*NLS + ls)*128 + row)*16 + j,   NLS = LR/16
+//  Step ls (16 wide) of tile vt: [mi][lane][8 bytes], bytes 2i, 2i+1 = pair i
+//  (same row/column rule as above with 16*ls in place of the k16 offset),
+//  stored offset-binary (code + 128).
+//    byte offset = (((vt*NLS + ls)*8 + mi)*32 + lane)*8,          NLS = LR/16
 //
 //  Correction row scales: [V_pad] fp16 bits (zero on padding rows).
 #pragma once
@@ -47,22 +46,23 @@ constexpr int kPrepassKSplit = 256;  // d per pre-pass block
 constexpr int64_t kDefaultWaitBudget = 2000000000LL;  // cycles, about one second
 
 struct DecodeParams {
-  CUtensorMap tmap_x;   // x [M_total][d] bf16, box 64 x 16 rows, 128-byte swizzle
-  CUtensorMap tmap_t;   // pre-pass operand T [M_total][2*LR] bf16, same box (unused when LR = 0)
+  CUtensorMap tmap_x;   // x [M_total][d] bf16, box 64 x 16 rows (kernel instances that stream x; M > 8)
   const uint8_t *codes;
   const uint16_t *scales;
   const uint8_t *lr_codes;
   const uint16_t *s_a;
   const uint16_t *x;    // hidden states [M_total][d] bf16 (this chunk starts at row m0)
+  const uint32_t *ts;   // t hi/lo fragments for this token chunk
   int64_t V;
-  int num_tiles, d, d_pad, G_pad, g, nls, nls_core, rcp, rrp;
+  int num_tiles, d, d_pad, G_pad, g, nls, nls_core;
   int M;                // tokens in this chunk (1..16)
   int m0;               // index of the chunk's first token
+  int NT;               // n-tiles of 8 tokens (1 or 2)
   void *out;            // logits [M_total][V] (NULL in CE mode)
   int out_fp32;
   // CE mode (out == NULL)
   const int32_t *targets;  // [M_total]
-  float2 *ce_part;         // [num_units * 4][M_total] (max, sum exp)
+  float2 *ce_part;         // [num_units][M_total] (max, sum exp)
   float *ce_tlogit;        // [M_total]
   int M_total;
   int *err;
@@ -137,8 +137,7 @@ cudaError_t launch_prepass_t(const PrepassParams &pp, const uint16_t *lr_t, int 
 size_t prepass_smem(int M);  // dynamic shared memory of one pre-pass block
 size_t prepass_partial_bytes(int M, int lr, int d);
 // pdl: launch as a programmatic dependent of the immediately preceding pre-pass grid.
-// Builds the x (and, when LR > 0, T) tensor maps from dp.x / T, then launches.
-cudaError_t launch_decode(const DecodeParams &dp, const uint16_t *T, int grid, cudaStream_t s, bool pdl);
+cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool pdl);
 // Tensor map of a bf16 [rows][cols] row-major matrix: box 64 columns x
 // box_rows rows, 128-byte swizzle, zero fill out of bounds.  False if the
 // driver entry point is missing or the encoder rejects the layout (base or

@@ -6,31 +6,35 @@
 
 namespace archead {
 
-// One thread per (row, 32-bit word) of a chunk: gather the word's 8 nibbles
-// from the canonical layout (byte j of a row = columns 2j (low nibble) and
-// 2j+1 (high nibble), two's complement).
+// One block per (vocabulary tile, 64-wide chunk of d): stage the canonical
+// 128 x 32 bytes in shared memory, then emit the 1024 fragment words.
 __global__ void build_res_codes_kernel(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst, int64_t V, int d,
                                        int d_pad) {
+  __shared__ uint8_t tile[kTileRows][kChunkK / 2];
   const int KC = d_pad / kChunkK;
-  const int64_t total = (int64_t)((V + kTileRows - 1) / kTileRows) * KC * kTileRows * 8;
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int q = (int)(e & 7);
-    const int r = (int)((e >> 3) % kTileRows);
-    const int64_t chunk = (e >> 3) / kTileRows;  // vt * KC + kc
-    const int kc = (int)(chunk % KC);
-    const int64_t vt = chunk / KC;
-    const int64_t row = vt * kTileRows + r;
+  const int vt = blockIdx.x / KC;
+  const int kc = blockIdx.x % KC;
+  for (int i = threadIdx.x; i < kTileRows * (kChunkK / 2); i += blockDim.x) {
+    int r = i / (kChunkK / 2), b = i % (kChunkK / 2);
+    int64_t row = (int64_t)vt * kTileRows + r;
+    // Padding rows and padding columns (k >= d; d is a multiple of 64) hold code 0.
+    tile[r][b] = (row < V && kc * kChunkK < d) ? src[row * (d / 2) + (int64_t)kc * (kChunkK / 2) + b] : (uint8_t)0;
+  }
+  __syncthreads();
+  uint32_t *out = reinterpret_cast<uint32_t *>(dst) + ((int64_t)vt * KC + kc) * 1024;
+  for (int w = threadIdx.x; w < 1024; w += blockDim.x) {
+    const int j = w & 3, lane = (w >> 2) & 31, mi = w >> 7;
+    const int gq = lane >> 2, cq = lane & 3;
     uint32_t word = 0;
     for (int p = 0; p < 8; ++p) {
-      const int k = kc * kChunkK + 8 * q + (p < 4 ? 2 * p : 2 * (p - 4) + 1);
-      uint32_t nib = 0;  // padding rows and columns (k >= d) hold code 0
-      if (row < V && k < d) {
-        const uint8_t byte = src[row * (d / 2) + k / 2];
-        nib = (k & 1) ? (byte >> 4) : (byte & 0xF);
-      }
+      const int i = p & 3, h = p >> 2;
+      const int r = mi * 16 + gq + 8 * (i & 1);
+      const int kl = j * 16 + 2 * cq + 8 * (i >> 1) + h;
+      const uint8_t byte = tile[r][kl >> 1];
+      const uint32_t nib = (kl & 1) ? (byte >> 4) : (byte & 0xF);
       word |= (nib ^ 0x8u) << (4 * p);  // two's complement -> offset binary
     }
-    reinterpret_cast<uint32_t *>(dst)[e] = word;
+    out[w] = word;
   }
 }
 
@@ -46,17 +50,18 @@ __global__ void build_res_scales_kernel(const uint16_t *__restrict__ src, uint16
   }
 }
 
-// One thread per byte of a (tile, 16-wide step) block.
+// One block per (tile, 16-wide step of the extended rank axis).
 __global__ void build_lr_codes_kernel(const int8_t *__restrict__ core_u, const int8_t *__restrict__ corr_a,
                                       uint8_t *__restrict__ dst, int64_t V, int rc, int rr, int rcp, int nls) {
-  const int64_t total = (int64_t)((V + kTileRows - 1) / kTileRows) * nls * kLrStepBytes;
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int j = (int)(e & 15);
-    const int r = (int)((e >> 4) % kTileRows);
-    const int64_t blk = (e >> 4) / kTileRows;  // vt * nls + ls
-    const int ls = (int)(blk % nls);
-    const int64_t row = (blk / nls) * kTileRows + r;
-    const int kk = ls * 16 + j;
+  const int vt = blockIdx.x / nls;
+  const int ls = blockIdx.x % nls;
+  uint8_t *out = dst + ((int64_t)vt * nls + ls) * kLrStepBytes;
+  for (int e = threadIdx.x; e < kLrStepBytes; e += blockDim.x) {
+    const int b = e & 7, lane = (e >> 3) & 31, mi = e >> 8;
+    const int gq = lane >> 2, cq = lane & 3;
+    const int i = b >> 1, h = b & 1;
+    const int64_t row = (int64_t)vt * kTileRows + mi * 16 + gq + 8 * (i & 1);
+    const int kk = ls * 16 + 2 * cq + 8 * (i >> 1) + h;
     int code = 0;
     if (row < V) {
       if (kk < rcp) {
@@ -65,7 +70,7 @@ __global__ void build_lr_codes_kernel(const int8_t *__restrict__ core_u, const i
         code = corr_a[row * rr + (kk - rcp)];
       }
     }
-    dst[e] = (uint8_t)(code + 128);
+    out[e] = (uint8_t)(code + 128);
   }
 }
 
@@ -97,10 +102,12 @@ __global__ void build_lr_t_kernel(const int8_t *__restrict__ q_v, const int8_t *
 cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, const uint16_t *res_scales,
                                  const int8_t *core_u, const int8_t *corr_a, const uint16_t *corr_a_scale,
                                  cudaStream_t s) {
-  build_res_codes_kernel<<<2048, 256, 0, s>>>(res_codes, p->codes, p->V, p->d, p->d_pad);
+  const int KC = p->d_pad / kChunkK;
+  build_res_codes_kernel<<<p->num_tiles * KC, 256, 0, s>>>(res_codes, p->codes, p->V, p->d, p->d_pad);
   build_res_scales_kernel<<<1024, 256, 0, s>>>(res_scales, p->scales, p->V, p->V_pad, p->G, p->G_pad);
   if (p->nls > 0)
-    build_lr_codes_kernel<<<1024, 256, 0, s>>>(core_u, corr_a, p->lr_codes, p->V, p->rc, p->rr, p->rcp, p->nls);
+    build_lr_codes_kernel<<<p->num_tiles * p->nls, 256, 0, s>>>(core_u, corr_a, p->lr_codes, p->V, p->rc, p->rr,
+                                                                 p->rcp, p->nls);
   build_row_scales_kernel<<<256, 256, 0, s>>>(p->rr > 0 ? corr_a_scale : nullptr, p->s_a, p->V, p->V_pad);
   if (p->lr > 0)
     build_lr_t_kernel<<<256, 256, 0, s>>>(p->q_v, p->q_b, p->lr_t, p->d, p->d_pad, p->rc, p->rr, p->rcp, p->lr);
@@ -119,6 +126,20 @@ struct DequantArgs {
   int d, d_pad, G_pad, g, rc, rr, rcp, nls;
 };
 
+// Position of (row-in-tile, column-in-16-step) inside a fragment: returns the
+// lane and sets pair index i and half h.
+__device__ __forceinline__ int frag_pos(int r, int k16, int &i, int &h) {
+  const int mrow = r & 15;
+  const int gq = mrow & 7;
+  const int ihi = k16 >> 3;
+  const int kp = k16 & 7;
+  i = (mrow >> 3) + 2 * ihi;
+  h = kp & 1;
+  return gq * 4 + (kp >> 1);
+}
+
+__device__ __forceinline__ float pair_half(uint32_t v, int h) { return h ? bf16_hi(v) : bf16_lo(v); }
+
 __global__ void debug_dequant_kernel(DequantArgs a, int comp, int64_t row0, int64_t nrows, float *out) {
   const int cols = comp == 0 ? a.d : ((comp == 1 || comp == 2) ? a.rc : a.rr);
   const int64_t total = nrows * cols;
@@ -129,27 +150,29 @@ __global__ void debug_dequant_kernel(DequantArgs a, int comp, int64_t row0, int6
     if (comp == 0 || comp == 1 || comp == 3) {
       const int64_t vt = row / kTileRows;
       const int r = (int)(row % kTileRows);
+      const int mi = r >> 4;
+      int i, h;
       if (comp == 0) {
-        // The word holding the column, unpacked as the prefill converter does.
         const int kc = col / kChunkK, kl = col % kChunkK;
+        const int j = kl >> 4;
+        const int lane = frag_pos(r, kl & 15, i, h);
         const int KC = a.d_pad / kChunkK;
-        const uint32_t w =
-            reinterpret_cast<const uint32_t *>(a.codes)[(((int64_t)vt * KC + kc) * kTileRows + r) * 8 + kl / 8];
+        const uint32_t w = reinterpret_cast<const uint32_t *>(
+            a.codes)[((((int64_t)vt * KC + kc) * 8 + mi) * 32 + lane) * 4 + j];
         uint32_t q[4];
-        unpack_int4x8(w, q);  // exact codes, pair i = columns (8q + 2i, 8q + 2i + 1)
+        unpack_int4x8_biased(w, q);  // the decode kernel's operands: 136 + code
         const int grp = col / a.g;
-        const uint32_t pr = q[(kl & 7) >> 1];
-        v = ((kl & 1) ? bf16_hi(pr) : bf16_lo(pr)) *
-            fp16_bits_to_f32(a.scales[((int64_t)vt * a.G_pad + grp) * kTileRows + r]);
+        v = (pair_half(q[i], h) - kInt4Bias) * fp16_bits_to_f32(a.scales[((int64_t)vt * a.G_pad + grp) * kTileRows + r]);
       } else {
         const int kk = comp == 1 ? col : a.rcp + col;
-        const int ls = kk >> 4, j = kk & 15;
-        const uint4 w4 = *reinterpret_cast<const uint4 *>(a.lr_codes + (((int64_t)vt * a.nls + ls) * kTileRows + r) * 16);
-        uint32_t q[8];
-        unpack_int8x16(w4, q);
-        const uint32_t pr = q[j >> 1];
+        const int ls = kk >> 4;
+        const int lane = frag_pos(r, kk & 15, i, h);
+        const uint2 w2 = *reinterpret_cast<const uint2 *>(
+            a.lr_codes + ((((int64_t)vt * a.nls + ls) * 8 + mi) * 32 + lane) * 8);
+        uint32_t q[4];
+        unpack_int8x8(w2.x, w2.y, q);
         const float sc = comp == 1 ? fp16_bits_to_f32(a.s_u[col]) : fp16_bits_to_f32(a.s_a[row]);
-        v = ((j & 1) ? bf16_hi(pr) : bf16_lo(pr)) * sc;
+        v = pair_half(q[i], h) * sc;
       }
     } else if (comp == 2) {
       v = (float)a.q_v[row * a.rc + col] * fp16_bits_to_f32(a.s_v[col]);

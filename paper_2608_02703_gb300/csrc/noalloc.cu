@@ -73,11 +73,11 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
     set_last_error_message("archead_forward_decode_noalloc: the decode kernel does not support this head shape");
     return ARCHEAD_ERR_UNSUPPORTED;
   }
-  // Scratch: [block counters | pre-pass partial sums | pre-pass operand T of the M tokens].
+  // Scratch: [block counters | pre-pass partial sums | rank-r fragments of one 16-token chunk].
   const int pairs = prepass_pairs((int)M, pack->lr);
   const size_t partial_bytes = (prepass_partial_bytes((int)M, pack->lr, pack->d) + 255) / 256 * 256;
-  const size_t t_bytes = (size_t)M * (pack->lr > 0 ? 2 * pack->lr : 64) * 2;
-  const size_t need = kNoallocCounterBytes + partial_bytes + t_bytes;
+  const size_t ts_bytes = (size_t)(pack->nls > 0 ? pack->nls : 1) * 1024;
+  const size_t need = kNoallocCounterBytes + partial_bytes + ts_bytes;
   if (need > kNoallocScratchBytes || (size_t)pairs * sizeof(int) > kNoallocCounterBytes) {
     set_last_error_message(
         "archead_forward_decode_noalloc: this head needs more scratch than the fixed 512 KiB array holds");
@@ -94,7 +94,7 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
   char *scratch = static_cast<char *>(base);
   int *counters = reinterpret_cast<int *>(scratch);
   float *partial = reinterpret_cast<float *>(scratch + kNoallocCounterBytes);
-  uint16_t *T = reinterpret_cast<uint16_t *>(scratch + kNoallocCounterBytes + partial_bytes);
+  uint32_t *ts = reinterpret_cast<uint32_t *>(scratch + kNoallocCounterBytes + partial_bytes);
 
   // The counters are the only state that must start at zero.
   e = cudaMemsetAsync(counters, 0, (size_t)pairs * sizeof(int), s);
@@ -116,8 +116,8 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
   pp.lr = pack->lr;
   pp.partial = partial;
   pp.counters = counters;
-  pp.ts = nullptr;
-  pp.T = T;
+  pp.ts = ts;
+  pp.T = nullptr;
   if (e == cudaSuccess) e = launch_prepass(pp, s, nullptr);  // no profiling events on this path
 
   DecodeParams dp{};
@@ -126,6 +126,7 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
   dp.lr_codes = pack->lr_codes;
   dp.s_a = pack->s_a;
   dp.x = static_cast<const uint16_t *>(x);
+  dp.ts = ts;
   dp.V = pack->V;
   dp.num_tiles = pack->num_tiles;
   dp.d = pack->d;
@@ -134,17 +135,16 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
   dp.g = pack->g;
   dp.nls = pack->nls;
   dp.nls_core = pack->nls_core;
-  dp.rcp = pack->rcp;
-  dp.rrp = pack->rrp;
   dp.M = (int)M;
   dp.m0 = 0;
+  dp.NT = M > 8 ? 2 : 1;
   dp.out = logits;
   dp.out_fp32 = out_dtype == ARCHEAD_OUT_FP32;
   dp.M_total = (int)M;
   dp.err = pack->err;
   dp.wait_budget = pack->wait_budget;
   const int units = decode_num_units(pack);
-  if (e == cudaSuccess) e = launch_decode(dp, T, units < pack->sm_count ? units : pack->sm_count, s, pack->lr > 0);
+  if (e == cudaSuccess) e = launch_decode(dp, units < pack->sm_count ? units : pack->sm_count, s, pack->lr > 0);
   if (e != cudaSuccess) {
     set_last_error_message(cudaGetErrorString(e));
     return ARCHEAD_ERR_CUDA;

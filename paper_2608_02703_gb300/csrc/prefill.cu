@@ -56,6 +56,82 @@ struct PrefillParams {
 // ------------------------------------------------------------------------
 // tcgen05 / TMA wrappers (inline PTX).
 // ------------------------------------------------------------------------
+__device__ __forceinline__ void tmem_alloc(uint32_t *slot, uint32_t cols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(slot)), "r"(cols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t cols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(taddr), "r"(cols) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory"); }
+
+__device__ __forceinline__ void tc_commit(uint64_t *bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                       uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// 32 lanes x 32 consecutive 32-bit columns starting at taddr (one value per column per thread).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// d0 += a * b0 and d1 += a * b1 as one packed fp32x2 FMA (round to nearest).
+__device__ __forceinline__ void fma2(float &d0, float &d1, float a, float b0, float b1) {
+  asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %2};\n mov.b64 rb, {%3, %4};\n mov.b64 rd, {%0, %1};\n"
+      " fma.rn.f32x2 rd, ra, rb, rd;\n mov.b64 {%0, %1}, rd;\n}\n"
+      : "+f"(d0), "+f"(d1)
+      : "f"(a), "f"(b0), "f"(b1));
+}
+
+// One step of the log-sum-exp merge: (m, s) of two disjoint sets -> of their union.
+__device__ __forceinline__ void lse_pair_merge(float am, float as, float bm, float bs, float &m, float &s) {
+  const float mx = fmaxf(am, bm), mn = fminf(am, bm);
+  const float e = mn == -INFINITY ? 0.f : __expf(mn - mx);
+  s = am >= bm ? fmaf(bs, e, as) : fmaf(as, e, bs);
+  m = mx;
+}
+
+// Shared-memory matrix descriptor: K-major operand in the 128-byte swizzle
+// layout (8-row groups of 128-byte rows, 1024 bytes apart).
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
+  uint64_t desc = 0;
+  desc |= (uint64_t)((saddr >> 4) & 0x3FFF);        // start address
+  desc |= (uint64_t)1 << 16;                        // leading byte offset (unused for this layout)
+  desc |= (uint64_t)(1024 >> 4) << 32;              // stride byte offset: 8 rows x 128 B
+  desc |= (uint64_t)1 << 46;                        // descriptor version (tcgen05)
+  desc |= (uint64_t)2 << 61;                        // 128-byte swizzle
+  return desc;
+}
+
+// Instruction descriptor: kind::f16, A = B = bf16, D = f32, K-major A and B.
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
 // Byte offset of bf16 element (row, k) in a 128-row x 64 K-major tile with the
 // 128-byte swizzle: 16-byte chunk k/8 of row r is stored at chunk (k/8) ^ (r%8).
 __device__ __forceinline__ uint32_t sw128_off(int row, int k) {
@@ -213,10 +289,8 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   } else if (warp < 8) {
     // ------------------------------ converters ------------------------------
     asm volatile("setmaxnreg.dec.sync.aligned.u32 88;\n" ::: "memory");
-    // One thread per row of the A tile: 32 bytes of INT4 codes (or 4 x 16
-    // bytes of INT8 codes) become 32 packed bf16 pairs in column order, stored
-    // as the row's eight 16-byte chunks of the 128-byte-swizzled tile.
-    const int r = (warp - 4) * 32 + lane;
+    const int cw = warp - 4;
+    const int gq = lane >> 2, cq = lane & 3;
     int s = 0;
     uint32_t ph = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
@@ -224,31 +298,38 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
         if (!mbar_wait_warp(&full[s], ph, p.wait_budget, abort_flag, p.err)) goto done;
         uint8_t *a_tile = smem + s * kPfStageBytes;
         const uint8_t *codes = a_tile + kPfABytes + kPfBBytes;
-        uint32_t a[32];
-        if (e < KC) {
-          const uint4 w0 = *reinterpret_cast<const uint4 *>(codes + r * 32);
-          const uint4 w1 = *reinterpret_cast<const uint4 *>(codes + r * 32 + 16);
-          const uint32_t ws[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            uint32_t u[4];
-            unpack_int4x8(ws[q], u);
+        for (int h = 0; h < 2; ++h) {
+          const int mi = cw * 2 + h;
+          if (e < KC) {
+            const uint4 w4 = *reinterpret_cast<const uint4 *>(codes + (mi * 32 + lane) * 16);
+            const uint32_t ws[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
-            for (int i = 0; i < 4; ++i) a[4 * q + i] = u[i];
-          }
-        } else {
+            for (int j = 0; j < 4; ++j) {
+              uint32_t a[4];
+              unpack_int4x8(ws[j], a);
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            uint32_t u[8];
-            unpack_int8x16(*reinterpret_cast<const uint4 *>(codes + q * kLrStepBytes + r * 16), u);
+              for (int i = 0; i < 4; ++i) {
+                const int row = mi * 16 + gq + 8 * (i & 1);
+                const int k = j * 16 + 2 * cq + 8 * (i >> 1);
+                *reinterpret_cast<uint32_t *>(a_tile + sw128_off(row, k)) = a[i];
+              }
+            }
+          } else {
 #pragma unroll
-            for (int i = 0; i < 8; ++i) a[8 * q + i] = u[i];
+            for (int q = 0; q < 4; ++q) {
+              const uint2 w2 = *reinterpret_cast<const uint2 *>(codes + q * kLrStepBytes + (mi * 32 + lane) * 8);
+              uint32_t a[4];
+              unpack_int8x8(w2.x, w2.y, a);
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                const int row = mi * 16 + gq + 8 * (i & 1);
+                const int k = q * 16 + 2 * cq + 8 * (i >> 1);
+                *reinterpret_cast<uint32_t *>(a_tile + sw128_off(row, k)) = a[i];
+              }
+            }
           }
         }
-#pragma unroll
-        for (int c = 0; c < 8; ++c)
-          *reinterpret_cast<uint4 *>(a_tile + sw128_off(r, 8 * c)) =
-              make_uint4(a[4 * c], a[4 * c + 1], a[4 * c + 2], a[4 * c + 3]);
         fence_proxy_async_smem();  // make the generic-proxy stores visible to the tensor core
         __syncwarp();
         if (lane == 0) mbar_arrive(&a_full[s]);
