@@ -1,0 +1,103 @@
+"""Full-size heads (the Qwen3-8B and Gemma-shaped configurations, the same
+seeded heads bench.py times) through the C ABI against the fp64 oracle:
+the whole vocabulary for decode token counts, sampled tokens for prefill
+(a token's logits depend on that token's hidden state only, so the oracle
+checks sampled rows exactly)."""
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_02703_gb300 import archead
+from synth import SHAPES, make_head, make_hidden, make_targets
+from tests import gpu_util as gu
+
+pytestmark = pytest.mark.gpu
+
+FULL = ("qwen3-8b", "gemma-4-e4b")
+PREFILL_M = {"qwen3-8b": 4096, "gemma-4-e4b": 2048}
+
+_state = {}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _build():
+    from paper_2608_02703_gb300.build import build
+
+    build()
+    yield
+    for pack, _ in _state.values():
+        pack.close()
+    _state.clear()
+
+
+def get(name):
+    if name not in _state:
+        shape = SHAPES[name]
+        head = make_head(shape, seed=0)
+        _state[name] = (archead.archead_pack_create(head, shape), head)
+    return _state[name]
+
+
+def _rows(y, idx):
+    return y[idx].float().cpu().numpy().astype(np.float64)
+
+
+@pytest.mark.parametrize("name", FULL)
+@pytest.mark.parametrize("M", [1, 16])
+def test_decode_full_vocabulary(name, M):
+    import torch
+
+    pack, head = get(name)
+    shape = SHAPES[name]
+    x = make_hidden(shape.d, M, seed=1, n_outliers=shape.n_outliers)
+    ref = oracle.logits(head, shape, x)
+    y = torch.full((M, shape.V), float("nan"), dtype=torch.float32, device="cuda")
+    archead.archead_forward(pack, gu.to_dev(x), M, y, archead.OUT_FP32)
+    assert archead.archead_sync_status(pack) == archead.OK
+    got = _rows(y, slice(None))
+    gu.check_logits(got, ref, where=f"{name} decode M={M}")
+    gu.check_argmax(got, ref, where=f"{name} decode M={M}")
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_decode_cross_entropy_full_vocabulary(name):
+    pack, head = get(name)
+    shape = SHAPES[name]
+    M = 16
+    x = make_hidden(shape.d, M, seed=2, n_outliers=shape.n_outliers)
+    t = make_targets(shape.V, M, seed=2)
+    ref = oracle.cross_entropy(head, shape, x, t)
+    ce, st = gu.forward_ce(pack, x, t)
+    assert st == archead.OK
+    assert np.max(np.abs(ce - ref["ce"])) <= gu.CE_ABS, f"{name}: CE max|d|={np.max(np.abs(ce - ref['ce'])):.3e}"
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_prefill_sampled_tokens(name):
+    """The bench's prefill launch (M = 4096 / 2048 tokens, logits and fused
+    CE), checked on sampled tokens: first and last of the 256-token tiles,
+    the ragged end and a few random ones."""
+    import torch
+
+    pack, head = get(name)
+    shape = SHAPES[name]
+    M = PREFILL_M[name]
+    x = make_hidden(shape.d, M, seed=1, n_outliers=shape.n_outliers)
+    t = make_targets(shape.V, M, seed=1)
+    rng = np.random.default_rng(7)
+    idx = np.unique(np.concatenate([[0, 1, 255, 256, 511, M // 2, M - 2, M - 1], rng.integers(0, M, 4)]))
+    ref = oracle.logits(head, shape, x[idx])
+    y = torch.empty((M, shape.V), dtype=torch.bfloat16, device="cuda")
+    archead.archead_forward(pack, gu.to_dev(x), M, y, archead.OUT_BF16)
+    assert archead.archead_sync_status(pack) == archead.OK
+    got = _rows(y, torch.from_numpy(idx).cuda())
+    gu.check_logits(got, ref, bf16=True, where=f"{name} prefill M={M} sampled")
+    gu.check_argmax(got, ref, where=f"{name} prefill M={M} sampled")
+    del y
+    ce, st = gu.forward_ce(pack, x, t)
+    assert st == archead.OK
+    ref_ce = oracle.cross_entropy(head, shape, x[idx], t[idx])
+    d = np.abs(ce[idx] - ref_ce["ce"])
+    assert np.max(d) <= gu.CE_ABS, f"{name}: prefill CE max|d|={np.max(d):.3e}"
+    assert np.all(np.isfinite(ce))
