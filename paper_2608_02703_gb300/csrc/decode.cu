@@ -278,7 +278,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
     if (threadIdx.x < kDecodeMaxTokens) tscale[threadIdx.x] = 1.f;
     asm volatile("bar.sync 1, %0;\n" ::"r"(kDecWarps * 32) : "memory");  // consumer warps only
   } else {
-    const bool ok = mbar_wait(xbar, 0, p.wait_budget, abort_flag, p.err);
+    const bool ok = mbar_wait_warp(xbar, 0, p.wait_budget, abort_flag, p.err);
     if (ok) {
       // Per-token power of two 2^-e that brings max |x| into [2^14, 2^15)
       // (fp16 range, and small tokens away from fp16 subnormals); tscale[m]
@@ -351,7 +351,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
     // once, so the producer can refill it while the warp computes.
     constexpr int NGS = GS <= SS ? SS / GS : 1;  // groups whose scales a stage carries
     for (int s = 0; s < res_stages; ++s) {
-      if (!mbar_wait(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
+      if (!mbar_wait_warp(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
       uint4 w[SC][kDecMT];
       float s_lo[NGS][kDecMT], s_hi[NGS][kDecMT];
       uint32_t bx[kStreamX ? SS : 1][NT][2];  // streamed x: this stage's B fragments
@@ -474,10 +474,10 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
         for (int c = 0; c < 4; ++c) part[a][b][c] = 0.f;
     for (int s = 0; s < lr_stages; ++s) {
       if (!t_ready) {
-        if (!mbar_wait(tbar, 0, p.wait_budget, abort_flag, p.err)) return;
+        if (!mbar_wait_warp(tbar, 0, p.wait_budget, abort_flag, p.err)) return;
         t_ready = true;
       }
-      if (!mbar_wait(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
+      if (!mbar_wait_warp(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
       const int ls0 = s * Geom::kLrSteps;
       const int nl = min(Geom::kLrSteps, p.nls - ls0);
       const bool last_stage = s == lr_stages - 1;
