@@ -33,13 +33,15 @@ constexpr int kSmemLimit = 227 * 1024;
 
 // 64-wide chunks of d per ring stage, by number of 8-token n-tiles.  The
 // shared-memory plan and the kernel instance launched both take it from here.
-__host__ __device__ constexpr int stage_chunks(int NT) { return NT == 1 ? 2 : 1; }
+__host__ __device__ constexpr int stage_chunks(int NT) { return 2; }
 
 // Instances with two n-tiles (9..16 tokens) do not keep the hidden states in
 // shared memory (16 rows of d would take most of it, leaving too shallow a
 // ring to stream at full bandwidth).  Each residual stage instead carries the
 // matching 64-wide chunks of x for 16 tokens, loaded by a 2-D TMA copy, and
-// those instances multiply bf16 operands (no fp16 staging).
+// those instances multiply bf16 operands (no fp16 staging).  Their warps read
+// codes and x from the stage as they compute and release it afterwards (the
+// registers to copy a stage out first are not there with two n-tiles).
 __host__ __device__ constexpr bool streams_x(int NT) { return NT == 2; }
 constexpr int kXChunkBytes = 16 * kChunkK * 2;  // 16 tokens x 64 of d, bf16, 128-byte swizzle
 
@@ -346,24 +348,27 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
 #pragma unroll
         for (int c = 0; c < 4; ++c) acc[a][b][c] = part[a][b][c] = 0.f;
 
-    // Residual: INT4 codes, promoted per group.  Each warp copies its share of
-    // a stage (codes and group scales) to registers and releases the slot at
-    // once, so the producer can refill it while the warp computes.
+    // Residual: INT4 codes, promoted per group.  With x resident, each warp
+    // copies its share of a stage (codes and group scales) to registers and
+    // releases the slot at once, so the producer can refill it while the warp
+    // computes; with x streamed, it releases the slot after its k steps.
     constexpr int NGS = GS <= SS ? SS / GS : 1;  // groups whose scales a stage carries
     for (int s = 0; s < res_stages; ++s) {
       if (!mbar_wait_warp(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
-      uint4 w[SC][kDecMT];
+      uint4 w[kStreamX ? 1 : SC][kDecMT];
       float s_lo[NGS][kDecMT], s_hi[NGS][kDecMT];
-      uint32_t bx[kStreamX ? SS : 1][NT][2];  // streamed x: this stage's B fragments
+      const uint8_t *sbuf = smem + (size_t)st * Geom::kBytes;
+      const uint8_t *cb = sbuf + tsel * SC * kChunkBytes + mi0 * 512 + lane * 16;
       if (active) {
-        const uint8_t *buf = smem + (size_t)st * Geom::kBytes;
-        const uint8_t *cb = buf + tsel * SC * kChunkBytes + mi0 * 512 + lane * 16;
-        const uint16_t *sc = reinterpret_cast<const uint16_t *>(buf + Geom::kCodeBytes + tsel * Geom::kScaleBytesPerTile) +
+        const uint16_t *sc = reinterpret_cast<const uint16_t *>(sbuf + Geom::kCodeBytes + tsel * Geom::kScaleBytesPerTile) +
                              mi0 * 16 + gq;
+        if (!kStreamX) {
 #pragma unroll
-        for (int c = 0; c < SC; ++c)
+          for (int c = 0; c < (kStreamX ? 1 : SC); ++c)
 #pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt) w[c][mt] = *reinterpret_cast<const uint4 *>(cb + c * kChunkBytes + mt * 512);
+            for (int mt = 0; mt < kDecMT; ++mt)
+              w[c][mt] = *reinterpret_cast<const uint4 *>(cb + c * kChunkBytes + mt * 512);
+        }
 #pragma unroll
         for (int gi = 0; gi < NGS; ++gi)
 #pragma unroll
@@ -371,27 +376,22 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
             s_lo[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16]);
             s_hi[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16 + 8]) * (kF16 ? 0.0625f : 1.f);  // fp16: x16
           }
-        if (kStreamX) {
-          // Token 8*nt + gq, k = 16*ks + 2*cq (+8): 128-byte rows, 16-byte
-          // chunk index XOR (row % 8) = gq.
-#pragma unroll
-          for (int ks = 0; ks < (kStreamX ? SS : 1); ++ks)
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-              const uint8_t *xr = buf + Geom::kXOff + (ks >> 2) * kXChunkBytes + (8 * nt + gq) * 128 + 4 * cq;
-              const int ch = 2 * (ks & 3);
-              bx[ks][nt][0] = *reinterpret_cast<const uint32_t *>(xr + ((ch ^ gq) << 4));
-              bx[ks][nt][1] = *reinterpret_cast<const uint32_t *>(xr + (((ch + 1) ^ gq) << 4));
-            }
-        }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&empty[st]);
+      const int st_done = st;
+      if (!kStreamX || !active) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[st]);
+      }
       if (++st == stages) st = 0, ph ^= 1;
       if (!active) continue;
       const int kbase = s * SS * 16;
 #pragma unroll
       for (int c = 0; c < SC; ++c) {
+        if (kStreamX) {
+#pragma unroll
+          for (int mt = 0; mt < kDecMT; ++mt)
+            w[0][mt] = *reinterpret_cast<const uint4 *>(cb + c * kChunkBytes + mt * 512);
+        }
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           const int ks = c * 4 + j;  // k step within the stage
@@ -399,8 +399,11 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
             if (kStreamX) {
-              b[nt][0] = bx[kStreamX ? ks : 0][nt][0];
-              b[nt][1] = bx[kStreamX ? ks : 0][nt][1];
+              // Token 8*nt + gq, k = 16*ks + 2*cq (+8): 128-byte rows, 16-byte
+              // chunk index XOR (row % 8) = gq.
+              const uint8_t *xr = sbuf + Geom::kXOff + c * kXChunkBytes + (8 * nt + gq) * 128 + 4 * cq;
+              b[nt][0] = *reinterpret_cast<const uint32_t *>(xr + (((2 * j) ^ gq) << 4));
+              b[nt][1] = *reinterpret_cast<const uint32_t *>(xr + (((2 * j + 1) ^ gq) << 4));
             } else {
               const uint16_t *q = xb[nt] + kbase + ks * 16;
               b[nt][0] = *reinterpret_cast<const uint32_t *>(q);
@@ -409,7 +412,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
           }
 #pragma unroll
           for (int mt = 0; mt < kDecMT; ++mt) {
-            const uint32_t word = j == 0 ? w[c][mt].x : j == 1 ? w[c][mt].y : j == 2 ? w[c][mt].z : w[c][mt].w;
+            const uint4 wv = w[kStreamX ? 0 : c][mt];
+            const uint32_t word = j == 0 ? wv.x : j == 1 ? wv.y : j == 2 ? wv.z : wv.w;
             uint32_t a[4];
             if (kF16)
               unpack_int4x8_f16(word, a);
@@ -450,6 +454,10 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
               promote_res<NT>(acc[mt], part[mt], s_lo[gi][mt], s_hi[gi][mt], nb_lo, nb_hi);
           }
         }
+      }
+      if (kStreamX) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[st_done]);
       }
     }
 
