@@ -184,6 +184,9 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
     // elected lane issues the copies: a single-lane loop issues bulk copies
     // several times more slowly.
     const bool leader = elect_one();
+    // The head is read once per forward: keep it from evicting the small
+    // data the pre-pass grid reads at the same time.
+    const uint64_t stream_policy = make_evict_first_policy();
     if (!kStreamX && leader) {
       mbar_arrive_expect_tx(xbar, (uint32_t)(p.M * p.d * 2));
       for (int m = 0; m < p.M; ++m)
@@ -221,9 +224,10 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
           }
           for (int t = 0; t < ntile; ++t) {
             const int64_t vt = (int64_t)kDecTiles * unit + t;
-            bulk_g2s(buf + t * SC * kChunkBytes, p.codes + (vt * KC + kc0) * kChunkBytes, SC * kChunkBytes, &full[st]);
-            bulk_g2s(buf + Geom::kCodeBytes + t * Geom::kScaleBytesPerTile, p.scales + (vt * p.G_pad + g0) * kTileRows,
-                     ng * kTileRows * 2, &full[st]);
+            bulk_g2s_hint(buf + t * SC * kChunkBytes, p.codes + (vt * KC + kc0) * kChunkBytes, SC * kChunkBytes,
+                          &full[st], stream_policy);
+            bulk_g2s_hint(buf + Geom::kCodeBytes + t * Geom::kScaleBytesPerTile, p.scales + (vt * p.G_pad + g0) * kTileRows,
+                          ng * kTileRows * 2, &full[st], stream_policy);
           }
         } else {
           const int ls0 = (s - res_stages) * Geom::kLrSteps;
@@ -232,8 +236,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
           mbar_arrive_expect_tx(&full[st], (uint32_t)(ntile * (nl * kLrStepBytes + (last ? kTileRows * 2 : 0))));
           for (int t = 0; t < ntile; ++t) {
             const int64_t vt = (int64_t)kDecTiles * unit + t;
-            bulk_g2s(buf + t * Geom::kLrSteps * kLrStepBytes, p.lr_codes + (vt * p.nls + ls0) * kLrStepBytes,
-                     nl * kLrStepBytes, &full[st]);
+            bulk_g2s_hint(buf + t * Geom::kLrSteps * kLrStepBytes, p.lr_codes + (vt * p.nls + ls0) * kLrStepBytes,
+                          nl * kLrStepBytes, &full[st], stream_policy);
             if (last)
               bulk_g2s(buf + Geom::kCodeBytes + t * Geom::kScaleBytesPerTile, p.s_a + vt * kTileRows, kTileRows * 2,
                        &full[st]);
