@@ -153,6 +153,25 @@ ARCHEAD_API archead_status archead_forward_ce_path(archead_pack *pack, const voi
                                        float *ce, archead_path path, void *stream);
 
 /*
+ * Greedy decoding output without logits: for each token m, index[m] = the
+ * vocabulary row of the largest logit of Eq. 7 (the first one on ties, as
+ * argmax) and, if value != NULL, value[m] = that logit (fp32, before any
+ * bf16 rounding).  The kernels keep a (largest logit, row) pair per token and
+ * vocabulary slice instead of writing the V-wide logits, and a second pass
+ * merges the slices in a fixed order.  The paper does not define this entry
+ * point; it is the generation-time use of the head (greedy next token).
+ *   x      device, bf16 [M][d] row-major, 16-byte aligned
+ *   index  device, int32 [M], 16-byte aligned (caller-owned)
+ *   value  device, float [M], 16-byte aligned, or NULL
+ * Returns ARCHEAD_ERR_INVALID_ARG for bad pointers or M < 0; M == 0 is a no-op.
+ * `path` as in archead_forward_path.
+ */
+ARCHEAD_API archead_status archead_forward_argmax(archead_pack *pack, const void *x, int64_t M, int32_t *index,
+                                                  float *value, void *stream);
+ARCHEAD_API archead_status archead_forward_argmax_path(archead_pack *pack, const void *x, int64_t M, int32_t *index,
+                                                       float *value, archead_path path, void *stream);
+
+/*
  * End-to-end call with HOST buffers: copies x (host, bf16 [M][d]) to the
  * device, runs archead_forward, copies the logits back to logits_host
  * ([M][V], bf16 or fp32) and waits for the stream.  Pinned host memory

@@ -39,7 +39,7 @@ EXPORTED = (
     "archead_forward_ce_path", "archead_forward_host", "archead_pack_bytes", "archead_device_bytes",
     "archead_debug_dequant", "archead_sync_status", "archead_set_wait_budget", "archead_debug_wait_timeout",
     "archead_profile_enable", "archead_profile_read", "archead_status_string", "archead_last_error",
-    "archead_forward_decode_noalloc",
+    "archead_forward_decode_noalloc", "archead_forward_argmax", "archead_forward_argmax_path",
 )
 
 
@@ -95,6 +95,8 @@ def load() -> ctypes.CDLL:
         "archead_forward_ce_path": (i32, [vp, vp, i64, vp, vp, i32, vp]),
         "archead_forward_host": (i32, [vp, vp, i64, vp, i32, vp]),
         "archead_forward_decode_noalloc": (i32, [vp, vp, i64, vp, i32, vp]),
+        "archead_forward_argmax": (i32, [vp, vp, i64, vp, vp, vp]),
+        "archead_forward_argmax_path": (i32, [vp, vp, i64, vp, vp, i32, vp]),
         "archead_pack_bytes": (i64, [vp]),
         "archead_device_bytes": (i64, [vp]),
         "archead_debug_dequant": (i32, [vp, i32, i64, i64, vp, vp]),
@@ -207,6 +209,17 @@ def archead_forward_ce_path(pack: Pack, x, M: int, targets, ce, path: int, strea
 def archead_forward_host(pack: Pack, x_host, M: int, logits_host, out_dtype: int = OUT_BF16, stream=None) -> None:
     _check(load().archead_forward_host(pack.handle, _ptr(x_host), M, _ptr(logits_host), out_dtype,
                                        _stream_ptr(stream)), "archead_forward_host")
+
+
+def archead_forward_argmax(pack: Pack, x, M: int, index, value=None, stream=None) -> None:
+    """Greedy next token per row of x: index (int32 [M]) and, optionally, its logit (fp32 [M])."""
+    _check(load().archead_forward_argmax(pack.handle, _ptr(x), M, _ptr(index), _ptr(value), _stream_ptr(stream)),
+           "archead_forward_argmax")
+
+
+def archead_forward_argmax_path(pack: Pack, x, M: int, index, value, path: int, stream=None) -> None:
+    _check(load().archead_forward_argmax_path(pack.handle, _ptr(x), M, _ptr(index), _ptr(value), path,
+                                              _stream_ptr(stream)), "archead_forward_argmax_path")
 
 
 def archead_forward_decode_noalloc(pack: Pack, x, M: int, logits, out_dtype: int = OUT_BF16, stream=None) -> None:

@@ -155,11 +155,13 @@ PrepassParams prepass_params(archead_pack *p, const void *x, int64_t M) {
   return pp;
 }
 
-// Decode path over M tokens, 16 at a time.  out == nullptr selects CE mode.
+// Decode path over M tokens, 16 at a time.  out == nullptr selects CE mode,
+// or greedy mode when amax_idx is given.
 archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
-                          const int32_t *targets, float *ce, cudaStream_t s) {
+                          const int32_t *targets, float *ce, int32_t *amax_idx, float *amax_val, cudaStream_t s) {
   if (!decode_supported(p->d_pad, p->nls, p->g)) return ARCHEAD_ERR_UNSUPPORTED;
   const bool ce_mode = out == nullptr;
+  const bool greedy = amax_idx != nullptr;
   ForwardPlan f = plan_decode(p, M, ce_mode);
   AH_CUDA(ensure_workspace(p, f.total, s));
   AH_CUDA(ensure_counters(p, prepass_pairs((int)M, p->lr), s));
@@ -187,6 +189,7 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   dp.out = out;
   dp.out_fp32 = out_fp32;
   dp.targets = targets;
+  dp.argmax = greedy;
   dp.ce_part = ce_mode ? at<float2>(p->ws, f.ce_part_off) : nullptr;
   dp.ce_tlogit = ce_mode ? at<float>(p->ws, f.tlogit_off) : nullptr;
   dp.M_total = (int)M;
@@ -209,8 +212,9 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   if (ce_mode) {
     cudaEvent_t ev = nullptr;
     timer_begin(p, "ce_finalize", s, &ev);
-    cudaError_t e = launch_ce_finalize(dp.ce_part, decode_num_units(p) * decode_parts_per_unit(), dp.ce_tlogit,
-                                       targets, p->V, (int)M, ce, p->err, s);
+    const int parts = decode_num_units(p) * decode_parts_per_unit();
+    cudaError_t e = greedy ? launch_argmax_finalize(dp.ce_part, parts, (int)M, amax_idx, amax_val, s)
+                           : launch_ce_finalize(dp.ce_part, parts, dp.ce_tlogit, targets, p->V, (int)M, ce, p->err, s);
     timer_end(p, "ce_finalize", s, ev);
     if (e != cudaSuccess) return cuda_status(e);
   }
@@ -218,10 +222,12 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
 }
 
 // Prefill path: rank-r pre-pass into the extended operand T, then the
-// tensor-core kernel.  out == nullptr selects CE mode.
+// tensor-core kernel.  out == nullptr selects CE mode, or greedy mode when
+// amax_idx is given.
 archead_status run_prefill(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
-                           const int32_t *targets, float *ce, cudaStream_t s) {
+                           const int32_t *targets, float *ce, int32_t *amax_idx, float *amax_val, cudaStream_t s) {
   const bool ce_mode = out == nullptr;
+  const bool greedy = amax_idx != nullptr;
   Carve c;
   const size_t t_off = c.take((size_t)M * std::max(2 * p->lr, 64) * 2);
   size_t ce_part_off = 0, tlogit_off = 0;
@@ -238,13 +244,14 @@ archead_status run_prefill(archead_pack *p, const void *x, int64_t M, void *out,
   float *tlogit = ce_mode ? at<float>(p->ws, tlogit_off) : nullptr;
   cudaEvent_t ev = nullptr;
   timer_begin(p, "prefill", s, &ev);
-  cudaError_t e = launch_prefill(p, x, (int)M, pp.T, out, out_fp32, targets, ce_part, tlogit, s);
+  cudaError_t e = launch_prefill(p, x, (int)M, pp.T, out, out_fp32, greedy, targets, ce_part, tlogit, s);
   timer_end(p, "prefill", s, ev);
   if (e != cudaSuccess) return cuda_status(e);
   if (ce_mode) {
     timer_begin(p, "ce_finalize", s, &ev);
-    e = launch_ce_finalize(ce_part, p->num_tiles * prefill_parts_per_vt(), tlogit, targets, p->V, (int)M, ce, p->err,
-                           s);
+    const int parts = p->num_tiles * prefill_parts_per_vt();
+    e = greedy ? launch_argmax_finalize(ce_part, parts, (int)M, amax_idx, amax_val, s)
+               : launch_ce_finalize(ce_part, parts, tlogit, targets, p->V, (int)M, ce, p->err, s);
     timer_end(p, "ce_finalize", s, ev);
     if (e != cudaSuccess) return cuda_status(e);
   }
@@ -252,13 +259,14 @@ archead_status run_prefill(archead_pack *p, const void *x, int64_t M, void *out,
 }
 
 archead_status run_forward(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
-                           const int32_t *targets, float *ce, archead_path path, cudaStream_t s) {
+                           const int32_t *targets, float *ce, archead_path path, cudaStream_t s,
+                           int32_t *amax_idx = nullptr, float *amax_val = nullptr) {
   if (path != ARCHEAD_PATH_AUTO && path != ARCHEAD_PATH_DECODE && path != ARCHEAD_PATH_PREFILL)
     return ARCHEAD_ERR_INVALID_ARG;
   AH_CUDA(cudaSetDevice(p->device));
   const bool decode = path == ARCHEAD_PATH_DECODE || (path == ARCHEAD_PATH_AUTO && M <= kDecodeMaxTokens);
-  if (decode) return run_decode(p, x, M, out, out_fp32, targets, ce, s);
-  return run_prefill(p, x, M, out, out_fp32, targets, ce, s);
+  if (decode) return run_decode(p, x, M, out, out_fp32, targets, ce, amax_idx, amax_val, s);
+  return run_prefill(p, x, M, out, out_fp32, targets, ce, amax_idx, amax_val, s);
 }
 
 }  // namespace
@@ -423,6 +431,19 @@ archead_status archead_forward_ce_path(archead_pack *pack, const void *x, int64_
 archead_status archead_forward_ce(archead_pack *pack, const void *x, int64_t M, const int32_t *targets, float *ce,
                                   void *stream) {
   return archead_forward_ce_path(pack, x, M, targets, ce, ARCHEAD_PATH_AUTO, stream);
+}
+
+archead_status archead_forward_argmax_path(archead_pack *pack, const void *x, int64_t M, int32_t *index,
+                                           float *value, archead_path path, void *stream) {
+  archead_status st = check_forward_args(pack, x, M, index);
+  if (st != ARCHEAD_OK || M == 0) return st;
+  if (value && !aligned16(value)) return ARCHEAD_ERR_INVALID_ARG;
+  return run_forward(pack, x, M, nullptr, 0, nullptr, nullptr, path, static_cast<cudaStream_t>(stream), index, value);
+}
+
+archead_status archead_forward_argmax(archead_pack *pack, const void *x, int64_t M, int32_t *index, float *value,
+                                      void *stream) {
+  return archead_forward_argmax_path(pack, x, M, index, value, ARCHEAD_PATH_AUTO, stream);
 }
 
 archead_status archead_forward_host(archead_pack *pack, const void *x_host, int64_t M, void *logits_host,

@@ -79,6 +79,45 @@ __global__ void __launch_bounds__(kCeWarps * 32) ce_finalize_wide_kernel(const f
   ce_store(acc, m, tlogit, targets, V, ce, err);
 }
 
+// Greedy decoding: merge the per-slice (value, row) partials of each token in
+// a fixed order (lanes over slices, then a fixed butterfly); ties keep the
+// lowest row, so the result is the first maximum as in argmax.
+__global__ void argmax_finalize_kernel(const float2 *__restrict__ part, int num_parts, int M,
+                                       int32_t *__restrict__ index, float *__restrict__ value) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (warp >= M) return;
+  float bv = -INFINITY;
+  int bi = 0x7fffffff;
+  for (int i = lane; i < num_parts; i += 32) {
+    const float2 v = part[(int64_t)i * M + warp];
+    const int vi = __float_as_int(v.y);
+    if (v.x > bv || (v.x == bv && vi < bi)) {
+      bv = v.x;
+      bi = vi;
+    }
+  }
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+    const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+    if (ov > bv || (ov == bv && oi < bi)) {
+      bv = ov;
+      bi = oi;
+    }
+  }
+  if (lane == 0) {
+    index[warp] = bi;
+    if (value) value[warp] = bv;
+  }
+}
+
+cudaError_t launch_argmax_finalize(const float2 *part, int num_parts, int M, int32_t *index, float *value,
+                                   cudaStream_t s) {
+  argmax_finalize_kernel<<<(M + 7) / 8, 256, 0, s>>>(part, num_parts, M, index, value);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_ce_finalize(const float2 *part, int num_parts, const float *tlogit, const int32_t *targets,
                                int64_t V, int M, float *ce, int *err, cudaStream_t s) {
   if (M >= 32) {

@@ -575,6 +575,39 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
               }
             }
       }
+    } else if (p.argmax) {
+      // Greedy partials: per (unit, warp, token) the largest logit and its
+      // row (the lowest row on ties), as (value, row bits).
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int tl = 0; tl < 2; ++tl) {
+          const int tok = nt * 8 + 2 * cq + tl;
+          float bv = -INFINITY;
+          int bi = 0x7fffffff;
+#pragma unroll
+          for (int mt = 0; mt < kDecMT; ++mt)
+#pragma unroll
+            for (int ih = 0; ih < 2; ++ih) {
+              const int64_t row = row_base + (mi0 + mt) * 16 + gq + 8 * ih;
+              const float v = acc[mt][nt][ih * 2 + tl];
+              if (active && row < p.V && (v > bv || (v == bv && (int)row < bi))) {
+                bv = v;
+                bi = (int)row;
+              }
+            }
+#pragma unroll
+          for (int off = 4; off < 32; off <<= 1) {
+            const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+            const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+            if (ov > bv || (ov == bv && oi < bi)) {
+              bv = ov;
+              bi = oi;
+            }
+          }
+          if (gq == 0 && tok < p.M)
+            p.ce_part[((int64_t)unit * kDecWarps + warp) * p.M_total + p.m0 + tok] = make_float2(bv, __int_as_float(bi));
+        }
     } else {
       // Cross-entropy partials: per (unit, warp, token) running max and sum of exp.
 #pragma unroll

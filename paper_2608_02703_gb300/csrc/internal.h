@@ -60,7 +60,8 @@ struct DecodeParams {
   int NT;               // n-tiles of 8 tokens (1 or 2)
   void *out;            // logits [M_total][V] (NULL in CE mode)
   int out_fp32;
-  // CE mode (out == NULL)
+  // CE mode (out == NULL, argmax == 0) or greedy mode (out == NULL, argmax != 0)
+  int argmax;
   const int32_t *targets;  // [M_total]
   float2 *ce_part;         // [num_units][M_total] (max, sum exp)
   float *ce_tlogit;        // [M_total]
@@ -147,8 +148,12 @@ int decode_num_units(const archead_pack *p);
 int decode_parts_per_unit();
 bool decode_supported(int d_pad, int nls, int g);
 cudaError_t launch_prefill(const archead_pack *pk, const void *x, int M, const uint16_t *T, void *out, int out_fp32,
-                           const int32_t *targets, float2 *ce_part, float *ce_tlogit, cudaStream_t s);
+                           bool argmax, const int32_t *targets, float2 *ce_part, float *ce_tlogit, cudaStream_t s);
 int prefill_parts_per_vt();
+// Greedy second pass: per token the largest (value, row) over the partials,
+// lowest row on ties.
+cudaError_t launch_argmax_finalize(const float2 *part, int num_parts, int M, int32_t *index, float *value,
+                                   cudaStream_t s);
 cudaError_t launch_ce_finalize(const float2 *part, int num_parts, const float *tlogit, const int32_t *targets,
                                int64_t V, int M, float *ce, int *err, cudaStream_t s);
 cudaError_t launch_wait_timeout_probe(int *err, int64_t budget, cudaStream_t s);

@@ -148,7 +148,7 @@ struct BlockPlan {
   __device__ int nblocks() const { return G_pad + (core_sub > 0) + (corr_sub > 0); }
 };
 
-template <int kMode>  // 0: logits, 1: cross-entropy partials
+template <int kMode>  // 0: logits, 1: cross-entropy partials, 2: greedy (largest logit, row) partials
 __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_constant__ PrefillParams p) {
   extern __shared__ uint8_t pf_smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(pf_smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -389,6 +389,50 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
               if (i < mcount) *o = __float2bfloat16_rn(acc[i]);
           }
         }
+      } else if (kMode == 2) {
+        // Greedy partials: the largest logit of each token over the warp's 32
+        // rows and its row (the lowest on ties), by the same token-halving
+        // butterfly as the cross entropy below: values in acc[0..63], rows
+        // (int bits) in acc[64..127]; lane L ends with tokens 4L..4L+3.
+        const int64_t rowbase = row - lane;
+        if (row >= p.V) {
+#pragma unroll
+          for (int i = 0; i < 128; ++i) acc[i] = -INFINITY;
+        }
+        {
+          const bool up = lane & 16;
+          const int my_row = (int)row, partner_row = (int)(rowbase + (lane ^ 16));
+#pragma unroll
+          for (int j = 0; j < 64; ++j) {
+            const float keep = up ? acc[j + 64] : acc[j];
+            const float give = up ? acc[j] : acc[j + 64];
+            const float recv = __shfl_xor_sync(0xffffffffu, give, 16);
+            const bool take = recv > keep || (recv == keep && partner_row < my_row);
+            acc[j] = take ? recv : keep;
+            acc[64 + j] = __int_as_float(take ? partner_row : my_row);
+          }
+        }
+#pragma unroll
+        for (int n = 64, o = 8; n > 4; n >>= 1, o >>= 1) {
+          const bool up = lane & o;
+#pragma unroll
+          for (int j = 0; j < n / 2; ++j) {
+            const float kv = up ? acc[j + n / 2] : acc[j];
+            const int ki = __float_as_int(up ? acc[64 + j + n / 2] : acc[64 + j]);
+            const float gv = up ? acc[j] : acc[j + n / 2];
+            const float gi = up ? acc[64 + j] : acc[64 + j + n / 2];
+            const float rv = __shfl_xor_sync(0xffffffffu, gv, o);
+            const int ri = __float_as_int(__shfl_xor_sync(0xffffffffu, gi, o));
+            const bool take = rv > kv || (rv == kv && ri < ki);
+            acc[j] = take ? rv : kv;
+            acc[64 + j] = __int_as_float(take ? ri : ki);
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int m = m0 + 4 * lane + j;
+          if (m < p.M) p.ce_part[((int64_t)vt * 4 + lg) * p.M + m] = make_float2(acc[j], acc[64 + j]);
+        }
       } else {
         // Target logits first: a token whose target is one of this warp's 32
         // rows takes its value from the owning lane (rare: about one token in
@@ -469,7 +513,7 @@ done:
 int prefill_parts_per_vt() { return 4; }
 
 cudaError_t launch_prefill(const archead_pack *pk, const void *x, int M, const uint16_t *T, void *out, int out_fp32,
-                           const int32_t *targets, float2 *ce_part, float *ce_tlogit, cudaStream_t s) {
+                           bool argmax, const int32_t *targets, float2 *ce_part, float *ce_tlogit, cudaStream_t s) {
   PrefillParams p{};
   if (!make_tma_map_bf16(&p.tmap_x, x, M, pk->d, 128)) return cudaErrorInvalidValue;
   const int kt = 2 * (pk->rcp + pk->rrp);
@@ -508,6 +552,14 @@ cudaError_t launch_prefill(const archead_pack *pk, const void *x, int M, const u
       attr = true;
     }
     prefill_kernel<0><<<grid, kPfThreads, kPfSmem, s>>>(p);
+  } else if (argmax) {
+    static bool attr = false;
+    if (!attr) {
+      cudaError_t e = cudaFuncSetAttribute(prefill_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPfSmem);
+      if (e != cudaSuccess) return e;
+      attr = true;
+    }
+    prefill_kernel<2><<<grid, kPfThreads, kPfSmem, s>>>(p);
   } else {
     static bool attr = false;
     if (!attr) {

@@ -73,3 +73,33 @@ def check_argmax(got: np.ndarray, ref: np.ndarray, where: str = "") -> int:
     bad = np.nonzero(sel & (a_got != a_ref))[0]
     assert bad.size == 0, f"{where}: argmax differs for tokens {bad[:8]}"
     return int(sel.sum())
+
+
+def forward_argmax(pack, x_bits: np.ndarray, path=archead.PATH_AUTO):
+    t = torch()
+    M = x_bits.shape[0]
+    idx = t.full((M,), -1, dtype=t.int32, device="cuda")
+    val = t.full((M,), float("nan"), dtype=t.float32, device="cuda")
+    archead.archead_forward_argmax_path(pack, to_dev(x_bits), M, idx, val, path)
+    assert archead.archead_sync_status(pack) == archead.OK
+    return idx.cpu().numpy().astype(np.int64), val.cpu().numpy().astype(np.float64)
+
+
+def check_greedy(idx: np.ndarray, val: np.ndarray, ref: np.ndarray, where: str = "") -> None:
+    """Greedy output against oracle logits: the index must be the oracle's
+    argmax wherever the top-2 gap exceeds ARGMAX_GAP, and must always name a
+    row whose oracle logit is within the logit bar of the maximum; the value
+    must be the logit of that row within the logit bar."""
+    rms = float(np.sqrt(np.mean(ref ** 2)))
+    tol = LOGIT_REL * rms
+    M = ref.shape[0]
+    assert np.all((idx >= 0) & (idx < ref.shape[1])), f"{where}: index out of range"
+    srt = np.sort(ref, axis=1)
+    gap = srt[:, -1] - srt[:, -2] if ref.shape[1] > 1 else np.full(M, np.inf)
+    a_ref = np.argmax(ref, axis=1)
+    sel = gap > ARGMAX_GAP
+    bad = np.nonzero(sel & (idx != a_ref))[0]
+    assert bad.size == 0, f"{where}: greedy index differs for tokens {bad[:8]}"
+    picked = ref[np.arange(M), idx]
+    assert np.all(srt[:, -1] - picked <= 2 * tol), f"{where}: greedy index names a row far below the maximum"
+    assert np.all(np.abs(val - picked) <= tol), f"{where}: greedy value max|d|={np.max(np.abs(val - picked)):.3e}"

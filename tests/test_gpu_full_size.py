@@ -74,9 +74,20 @@ def test_decode_cross_entropy_full_vocabulary(name):
 
 
 @pytest.mark.parametrize("name", FULL)
+def test_greedy_full_vocabulary(name):
+    pack, head = get(name)
+    shape = SHAPES[name]
+    M = 16
+    x = make_hidden(shape.d, M, seed=3, n_outliers=shape.n_outliers)
+    ref = oracle.logits(head, shape, x)
+    idx, val = gu.forward_argmax(pack, x)
+    gu.check_greedy(idx, val, ref, where=f"{name} greedy M={M}")
+
+
+@pytest.mark.parametrize("name", FULL)
 def test_prefill_sampled_tokens(name):
-    """The bench's prefill launch (M = 4096 / 2048 tokens, logits and fused
-    CE), checked on sampled tokens: first and last of the 256-token tiles,
+    """The bench's prefill launch (M = 4096 / 2048 tokens: logits, greedy
+    output and fused CE), checked on sampled tokens: first and last of the 256-token tiles,
     the ragged end and a few random ones."""
     import torch
 
@@ -95,6 +106,8 @@ def test_prefill_sampled_tokens(name):
     gu.check_logits(got, ref, bf16=True, where=f"{name} prefill M={M} sampled")
     gu.check_argmax(got, ref, where=f"{name} prefill M={M} sampled")
     del y
+    gi, gv = gu.forward_argmax(pack, x)
+    gu.check_greedy(gi[idx], gv[idx], ref, where=f"{name} prefill greedy M={M} sampled")
     ce, st = gu.forward_ce(pack, x, t)
     assert st == archead.OK
     ref_ce = oracle.cross_entropy(head, shape, x[idx], t[idx])

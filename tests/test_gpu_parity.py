@@ -117,6 +117,18 @@ def test_logits_many_tokens(name, M):
         gu.check_argmax(got, ref, where=f"{name} M={M} path={path}")
 
 
+@pytest.mark.parametrize("name", ["ragged", "tiny", "g32", "g256", "corr_only", "one_row", "max_rank"])
+@pytest.mark.parametrize("M", [1, 7, 16, 40])
+def test_greedy(name, M):
+    pack, head = get(name)
+    shape = SHAPES[name]
+    x = make_hidden(shape.d, M, seed=300 + M)
+    ref = oracle.logits(head, shape, x)
+    for path in (archead.PATH_AUTO, archead.PATH_DECODE, archead.PATH_PREFILL):
+        idx, val = gu.forward_argmax(pack, x, path)
+        gu.check_greedy(idx, val, ref, where=f"{name} M={M} path={path}")
+
+
 @pytest.mark.parametrize("name", ["ragged", "tiny", "g32", "g256", "corr_only", "one_row"])
 @pytest.mark.parametrize("M", [1, 5, 16, 33])
 def test_cross_entropy(name, M):
