@@ -41,13 +41,17 @@ class _Head(ctypes.Structure):
     _fields_ = [
         ("V", ctypes.c_int64), ("d", ctypes.c_int64),
         ("core_rank", ctypes.c_int32), ("corr_rank", ctypes.c_int32),
-        ("group_size", ctypes.c_int32), ("pad_", ctypes.c_int32),
+        ("group_size", ctypes.c_int32), ("format", ctypes.c_int32),
         ("res_codes", ctypes.c_void_p), ("res_scales", ctypes.c_void_p),
         ("core_u", ctypes.c_void_p), ("core_u_scale", ctypes.c_void_p),
         ("core_v", ctypes.c_void_p), ("core_v_scale", ctypes.c_void_p),
         ("corr_a", ctypes.c_void_p), ("corr_a_scale", ctypes.c_void_p),
         ("corr_b", ctypes.c_void_p), ("corr_b_scale", ctypes.c_void_p),
+        ("res_scale_codes", ctypes.c_void_p), ("res_row_scale", ctypes.c_void_p),
+        ("core_u5", ctypes.c_void_p),
     ]
+
+FORMATS = {"int8": 0, "sc4": 1}
 
 
 def use_library(path: Optional[str]) -> None:
@@ -76,12 +80,16 @@ def _configure(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.oracle_fp16_values.argtypes = [vp, i64, vp]
     lib.oracle_bf16_values.argtypes = [vp, i64, vp]
     lib.oracle_unpack_int4.argtypes = [vp, i64, vp]
+    lib.oracle_unpack_int5.argtypes = [vp, i64, i64, vp]
+    lib.oracle_unpack_scale_codes.argtypes = [vp, i64, i64, vp]
     lib.oracle_dequant_rows.argtypes = [ctypes.POINTER(_Head), i64, i64, vp]
     lib.oracle_component.argtypes = [ctypes.POINTER(_Head), ctypes.c_int, i64, i64, vp]
     lib.oracle_logits.argtypes = [ctypes.POINTER(_Head), vp, i64, i64, i64, vp]
     lib.oracle_ce.argtypes = [ctypes.POINTER(_Head), vp, i64, vp, vp, vp, vp, vp]
     lib.oracle_packed_bytes.restype = i64
     lib.oracle_packed_bytes.argtypes = [i64, i64, i64, i64, i64]
+    lib.oracle_packed_bytes_sc4.restype = i64
+    lib.oracle_packed_bytes_sc4.argtypes = [i64, i64, i64, i64, i64]
     lib.oracle_dense_bf16_bytes.restype = i64
     lib.oracle_dense_bf16_bytes.argtypes = [i64, i64]
     lib.oracle_threads.restype = ctypes.c_int
@@ -95,10 +103,21 @@ def _ptr(a: np.ndarray) -> int:
 
 
 def _head_struct(head: Dict[str, np.ndarray], shape) -> _Head:
-    need = {
+    fmt = getattr(shape, "fmt", "int8")
+    G = shape.d // shape.group_size
+    if fmt == "sc4":
+        need = {
+            "res_scale_codes": (np.uint8, (shape.V, (G + 1) // 2)),
+            "res_row_scale": (np.uint16, (shape.V,)),
+            "core_u5": (np.uint8, (shape.V, (5 * shape.core_rank + 7) // 8)),
+        }
+    else:
+        need = {
+            "res_scales": (np.uint16, (shape.V, G)),
+            "core_u": (np.int8, (shape.V, shape.core_rank)),
+        }
+    need.update({
         "res_codes": (np.uint8, (shape.V, shape.d // 2)),
-        "res_scales": (np.uint16, (shape.V, shape.d // shape.group_size)),
-        "core_u": (np.int8, (shape.V, shape.core_rank)),
         "core_u_scale": (np.uint16, (shape.core_rank,)),
         "core_v": (np.int8, (shape.d, shape.core_rank)),
         "core_v_scale": (np.uint16, (shape.core_rank,)),
@@ -106,9 +125,9 @@ def _head_struct(head: Dict[str, np.ndarray], shape) -> _Head:
         "corr_a_scale": (np.uint16, (shape.V,)),
         "corr_b": (np.int8, (shape.d, shape.corr_rank)),
         "corr_b_scale": (np.uint16, (shape.d // shape.group_size, shape.corr_rank)),
-    }
+    })
     h = _Head(V=shape.V, d=shape.d, core_rank=shape.core_rank, corr_rank=shape.corr_rank,
-              group_size=shape.group_size, pad_=0)
+              group_size=shape.group_size, format=FORMATS[fmt])
     for name, (dt, shp) in need.items():
         a = head[name]
         if a.dtype != dt or tuple(a.shape) != shp or not a.flags["C_CONTIGUOUS"]:
@@ -137,6 +156,24 @@ def unpack_int4(packed: np.ndarray) -> np.ndarray:
     out = np.empty(packed.size * 2, dtype=np.int8)
     _load().oracle_unpack_int4(_ptr(packed), packed.size * 2, _ptr(out))
     return out.reshape(packed.shape[:-1] + (packed.shape[-1] * 2,)) if packed.ndim else out
+
+
+def unpack_int5(packed: np.ndarray, rank: int) -> np.ndarray:
+    """Signed 5-bit codes [rows, rank] of rows of ceil(5 rank / 8) packed bytes."""
+    packed = np.ascontiguousarray(packed, dtype=np.uint8)
+    rows = packed.shape[0]
+    out = np.empty((rows, rank), dtype=np.int8)
+    _load().oracle_unpack_int5(_ptr(packed), rows, rank, _ptr(out))
+    return out
+
+
+def unpack_scale_codes(packed: np.ndarray, groups: int) -> np.ndarray:
+    """4-bit unsigned group-scale codes [rows, groups] (two per byte, low nibble first)."""
+    packed = np.ascontiguousarray(packed, dtype=np.uint8)
+    rows = packed.shape[0]
+    out = np.empty((rows, groups), dtype=np.int8)
+    _load().oracle_unpack_scale_codes(_ptr(packed), rows, groups, _ptr(out))
+    return out
 
 
 def dequant_rows(head, shape, row0: int = 0, nrows: Optional[int] = None) -> np.ndarray:
@@ -204,7 +241,8 @@ def cross_entropy(head, shape, x_bits: np.ndarray, targets: np.ndarray, chunk: i
 
 def packed_bytes(shape) -> int:
     """Eq. 10 of the paper over the stored components of this packed format."""
-    return int(_load().oracle_packed_bytes(shape.V, shape.d, shape.core_rank, shape.corr_rank, shape.group_size))
+    fn = _load().oracle_packed_bytes_sc4 if getattr(shape, "fmt", "int8") == "sc4" else _load().oracle_packed_bytes
+    return int(fn(shape.V, shape.d, shape.core_rank, shape.corr_rank, shape.group_size))
 
 
 def dense_bf16_bytes(V: int, d: int) -> int:

@@ -23,6 +23,16 @@
  *  - All quantisers are symmetric (no zero points); scales are IEEE fp16.
  *  - A_w is quantised per row (one scale per vocabulary row) and B_w per
  *    (d-group of size g, rank column); the core factors per column.
+ *
+ * Two stored formats.  "int8" (format 0): INT8 core left codes and one fp16
+ * scale per residual group.  "sc4" (format 1), the paper's own format
+ * (Section 3.2, Eq. 3: Q_5 core left factor, SC4 residual with quantised
+ * group scales; Appendix C, packed state dictionary):
+ *  - core left codes are 5-bit two's complement (-16..15); row n stores its
+ *    r_c codes in ceil(5 r_c / 8) bytes, code j in bits 5j..5j+4 of the row's
+ *    bytes taken as one little-endian bit string;
+ *  - a residual group scale is s_row[n] * (q + 1), with q a 4-bit unsigned
+ *    code (two per byte, low nibble = even group) and s_row one fp16 per row.
  */
 #include <math.h>
 #include <stdint.h>
@@ -34,10 +44,10 @@
 
 typedef struct {
   int64_t V, d;
-  int32_t core_rank, corr_rank, group_size, pad_;
+  int32_t core_rank, corr_rank, group_size, format; /* format: 0 int8, 1 sc4 */
   const uint8_t *res_codes;      /* V x d/2                       */
-  const uint16_t *res_scales;    /* V x d/g   fp16 bits           */
-  const int8_t *core_u;          /* V x r_c                       */
+  const uint16_t *res_scales;    /* V x d/g   fp16 bits   (int8)  */
+  const int8_t *core_u;          /* V x r_c               (int8)  */
   const uint16_t *core_u_scale;  /* r_c       fp16 bits           */
   const int8_t *core_v;          /* d x r_c                       */
   const uint16_t *core_v_scale;  /* r_c       fp16 bits           */
@@ -45,6 +55,9 @@ typedef struct {
   const uint16_t *corr_a_scale;  /* V         fp16 bits           */
   const int8_t *corr_b;          /* d x r_r                       */
   const uint16_t *corr_b_scale;  /* d/g x r_r fp16 bits           */
+  const uint8_t *res_scale_codes; /* V x ceil(G/2), 4-bit codes (sc4) */
+  const uint16_t *res_row_scale;  /* V         fp16 bits     (sc4) */
+  const uint8_t *core_u5;         /* V x ceil(5 r_c/8)       (sc4) */
 } oracle_head;
 
 /* IEEE-754 binary16: 1 sign bit, 5 exponent bits (bias 15), 10 fraction bits. */
@@ -86,6 +99,51 @@ int oracle_int4_code(const uint8_t *row, int64_t k) {
   return nib >= 8 ? nib - 16 : nib;
 }
 
+/* Signed 5-bit code j of a row of packed bytes: bits 5j..5j+4, bit b of the
+ * row being bit b%8 of byte b/8; two's complement over 5 bits. */
+int oracle_int5_code(const uint8_t *row, int64_t j) {
+  int v = 0;
+  for (int b = 0; b < 5; ++b) {
+    int64_t bit = 5 * j + b;
+    v |= ((row[bit / 8] >> (bit % 8)) & 1) << b;
+  }
+  return v >= 16 ? v - 32 : v;
+}
+
+/* 4-bit unsigned group-scale code of group grp: byte grp/2, low nibble for even grp. */
+int oracle_scale_code(const uint8_t *row, int64_t grp) {
+  int byte = row[grp / 2];
+  return (grp % 2 == 0) ? (byte & 0x0F) : ((byte >> 4) & 0x0F);
+}
+
+/* Residual group scale s_R[n, grp] of either format. */
+static double res_scale(const oracle_head *h, int64_t n, int64_t grp) {
+  const int64_t G = h->d / h->group_size;
+  if (h->format == 1) {
+    const int64_t nb = (G + 1) / 2;
+    return oracle_fp16_value(h->res_row_scale[n]) * (double)(oracle_scale_code(h->res_scale_codes + n * nb, grp) + 1);
+  }
+  return oracle_fp16_value(h->res_scales[n * G + grp]);
+}
+
+/* Core left code qU[n, j] of either format. */
+static int core_u_code(const oracle_head *h, int64_t n, int j) {
+  if (h->format == 1) return oracle_int5_code(h->core_u5 + n * ((5 * (int64_t)h->core_rank + 7) / 8), j);
+  return h->core_u[n * h->core_rank + j];
+}
+
+void oracle_unpack_int5(const uint8_t *in, int64_t rows, int64_t rank, int8_t *out) {
+  const int64_t nb = (5 * rank + 7) / 8;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t j = 0; j < rank; ++j) out[r * rank + j] = (int8_t)oracle_int5_code(in + r * nb, j);
+}
+
+void oracle_unpack_scale_codes(const uint8_t *in, int64_t rows, int64_t groups, int8_t *out) {
+  const int64_t nb = (groups + 1) / 2;
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t j = 0; j < groups; ++j) out[r * groups + j] = (int8_t)oracle_scale_code(in + r * nb, j);
+}
+
 void oracle_fp16_values(const uint16_t *in, int64_t n, double *out) {
   for (int64_t i = 0; i < n; ++i) out[i] = oracle_fp16_value(in[i]);
 }
@@ -102,6 +160,7 @@ static int check_head(const oracle_head *h) {
   if (!h || h->V < 1 || h->d < 2 || h->group_size < 1) return -1;
   if (h->d % 2 != 0 || h->d % h->group_size != 0) return -1;
   if (h->core_rank < 0 || h->corr_rank < 0) return -1;
+  if (h->format != 0 && h->format != 1) return -1;
   return 0;
 }
 
@@ -148,13 +207,12 @@ static int make_cache(const oracle_head *h, side_cache *c) {
 static void dequant_row(const oracle_head *h, const side_cache *c, int64_t n, double *w, double *u, double *a) {
   const int64_t d = h->d;
   const int g = h->group_size, rc = h->core_rank, rr = h->corr_rank;
-  const int64_t G = d / g;
   const uint8_t *codes = h->res_codes + n * (d / 2);
-  for (int j = 0; j < rc; ++j) u[j] = (double)h->core_u[n * rc + j] * c->su[j];
+  for (int j = 0; j < rc; ++j) u[j] = (double)core_u_code(h, n, j) * c->su[j];
   double s_a = rr > 0 ? oracle_fp16_value(h->corr_a_scale[n]) : 0.0;
   for (int j = 0; j < rr; ++j) a[j] = (double)h->corr_a[n * rr + j] * s_a;
   for (int64_t k = 0; k < d; ++k) {
-    double s_r = oracle_fp16_value(h->res_scales[n * G + k / g]);
+    double s_r = res_scale(h, n, k / g);
     double v = (double)oracle_int4_code(codes, k) * s_r;
     double core = 0.0;
     for (int j = 0; j < rc; ++j) core += u[j] * c->vdq[k * rc + j];
@@ -206,18 +264,16 @@ int oracle_component(const oracle_head *h, int comp, int64_t row0, int64_t nrows
   if (check_head(h) || row0 < 0 || nrows < 0) return -1;
   const int64_t d = h->d;
   const int g = h->group_size, rc = h->core_rank, rr = h->corr_rank;
-  const int64_t G = d / g;
   int64_t limit = (comp == 2 || comp == 4) ? d : h->V;
   if (comp < 0 || comp > 4 || row0 + nrows > limit) return -1;
   for (int64_t i = 0; i < nrows; ++i) {
     int64_t r = row0 + i;
     if (comp == 0) {
       for (int64_t k = 0; k < d; ++k)
-        out[i * d + k] = (double)oracle_int4_code(h->res_codes + r * (d / 2), k) *
-                         oracle_fp16_value(h->res_scales[r * G + k / g]);
+        out[i * d + k] = (double)oracle_int4_code(h->res_codes + r * (d / 2), k) * res_scale(h, r, k / g);
     } else if (comp == 1) {
       for (int j = 0; j < rc; ++j)
-        out[i * rc + j] = (double)h->core_u[r * rc + j] * oracle_fp16_value(h->core_u_scale[j]);
+        out[i * rc + j] = (double)core_u_code(h, r, j) * oracle_fp16_value(h->core_u_scale[j]);
     } else if (comp == 2) {
       for (int j = 0; j < rc; ++j)
         out[i * rc + j] = (double)h->core_v[r * rc + j] * oracle_fp16_value(h->core_v_scale[j]);
@@ -340,6 +396,28 @@ int64_t oracle_packed_bytes(int64_t V, int64_t d, int64_t rc, int64_t rr, int64_
   if (rr > 0) bytes += V * 2; /* correction row scales (absent when r_r = 0) */
   bytes += d * rr;         /* correction right codes*/
   bytes += G * rr * 2;     /* correction group scales */
+  return bytes;
+}
+
+/*
+ * The same sum for the sc4 format: 4-bit group-scale codes (two per byte)
+ * plus one fp16 row scale replace the fp16 group scales, and the core left
+ * factor takes ceil(5 r_c / 8) bytes per row.
+ */
+int64_t oracle_packed_bytes_sc4(int64_t V, int64_t d, int64_t rc, int64_t rr, int64_t g) {
+  int64_t G = d / g;
+  int64_t bytes = 0;
+  bytes += V * d / 2;            /* residual codes                  */
+  bytes += V * ((G + 1) / 2);    /* residual group-scale codes      */
+  bytes += V * 2;                /* residual row scales             */
+  bytes += V * ((5 * rc + 7) / 8); /* core left codes, 5-bit        */
+  bytes += rc * 2;               /* core left scales                */
+  bytes += d * rc;               /* core right codes                */
+  bytes += rc * 2;               /* core right scales               */
+  bytes += V * rr;               /* correction left codes           */
+  if (rr > 0) bytes += V * 2;    /* correction row scales           */
+  bytes += d * rr;               /* correction right codes          */
+  bytes += G * rr * 2;           /* correction group scales         */
   return bytes;
 }
 

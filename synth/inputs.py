@@ -19,6 +19,21 @@ dictionary") in the symmetric INT8/INT4 variant used by this library:
     corr_b_scale  uint16 [d/g, r_r]  fp16, one per (d-group, column)
                                      (group-wise INT8 along d)
 
+The paper's own packed format (Section 3.2, Eq. 3: a 5-bit core left
+factor and the SC4 residual with quantised group scales; Appendix C) is the
+"sc4" variant.  It changes three arrays and keeps the rest:
+
+    res_scale_codes uint8 [V, ceil(G/2)]  4-bit unsigned group-scale codes q,
+                                          two per byte, low nibble = even
+                                          group; the group scale is
+                                          res_row_scale[n] * (q + 1)
+    res_row_scale   uint16 [V]            fp16, one per row
+    core_u5         uint8 [V, ceil(5 r_c / 8)]  5-bit two's complement core
+                                          left codes (-16..15); code j of a
+                                          row is bits 5j..5j+4 of the row's
+                                          bytes read as one little-endian
+                                          bit string; unused top bits zero
+
 Hidden states follow the anisotropic recipe x = z diag(s) Q with s
 log-spaced over [1e-2, 1e1], Q a Haar-random orthogonal matrix and a few
 outlier channels scaled by 20, cast to bf16 (round to nearest even).  The
@@ -47,10 +62,21 @@ class HeadShape:
     corr_rank: int
     group_size: int
     n_outliers: int = 4
+    fmt: str = "int8"  # "int8": INT8 core, fp16 group scales; "sc4": the paper's packed format
 
     @property
     def groups(self) -> int:
         return self.d // self.group_size
+
+    @property
+    def core_u5_bytes(self) -> int:
+        """Bytes per row of the 5-bit core left factor (sc4)."""
+        return (5 * self.core_rank + 7) // 8
+
+    @property
+    def scale_code_bytes(self) -> int:
+        """Bytes per row of the 4-bit group-scale codes (sc4)."""
+        return (self.groups + 1) // 2
 
 
 # Head shapes of the paper's models (Section 4, "Models") in this library's
@@ -59,6 +85,10 @@ SHAPES: Dict[str, HeadShape] = {
     "tiny": HeadShape(V=4096, d=512, core_rank=64, corr_rank=16, group_size=64, n_outliers=4),
     "qwen3-8b": HeadShape(V=151936, d=4096, core_rank=128, corr_rank=32, group_size=128, n_outliers=4),
     "gemma-4-e4b": HeadShape(V=262144, d=2560, core_rank=128, corr_rank=32, group_size=128, n_outliers=8),
+    # The paper's packed format with its Qwen hyper-parameters (Section 4,
+    # "Baselines and implementation": r_c = 10, r_r = 6, groups of 64).
+    "tiny-sc4": HeadShape(V=4096, d=512, core_rank=10, corr_rank=6, group_size=64, n_outliers=4, fmt="sc4"),
+    "qwen3-8b-sc4": HeadShape(V=151936, d=4096, core_rank=10, corr_rank=6, group_size=64, n_outliers=4, fmt="sc4"),
 }
 
 # Element rms targets of the three parts of the head.  The paper prints no
@@ -69,6 +99,9 @@ _RMS_CORRECTION = 0.0012
 # rms of a code drawn uniformly from [-8, 7] and from [-127, 127]
 _RMS_INT4 = float(np.sqrt(np.mean(np.arange(-8, 8, dtype=np.float64) ** 2)))
 _MS_INT8 = float(np.mean(np.arange(-127, 128, dtype=np.float64) ** 2))
+_MS_INT5 = float(np.mean(np.arange(-16, 16, dtype=np.float64) ** 2))
+# rms of the group-scale multiplier q + 1 for q uniform over [0, 15]
+_RMS_SCALE_MULT = float(np.sqrt(np.mean(np.arange(1, 17, dtype=np.float64) ** 2)))
 
 _HEAD_STREAMS = (
     "res_codes", "res_scales", "core_u", "core_u_scale", "core_v", "core_v_scale",
@@ -91,8 +124,22 @@ def _int8_codes(rng: np.random.Generator, shape) -> np.ndarray:
     return rng.integers(-127, 128, size=shape, dtype=np.int8)
 
 
+def _uniform_bits(rng: np.random.Generator, rows: int, nbytes: int, used_bits: int) -> np.ndarray:
+    """Uniform random bytes [rows, nbytes] with the bits past used_bits of
+    each row zero: every field of the row is then uniform over its range."""
+    b = rng.integers(0, 256, size=(rows, nbytes), dtype=np.uint8)
+    spare = 8 * nbytes - used_bits
+    if nbytes and spare:
+        b[:, -1] &= np.uint8((1 << (8 - spare)) - 1)
+    return b
+
+
 def make_head(shape: HeadShape, seed: int = 0) -> Dict[str, np.ndarray]:
     """Draw one packed head in the canonical layout described above."""
+    if shape.fmt == "sc4":
+        return _make_head_sc4(shape, seed)
+    if shape.fmt != "int8":
+        raise ValueError(f"unknown packed format {shape.fmt!r}")
     V, d, rc, rr, g = shape.V, shape.d, shape.core_rank, shape.corr_rank, shape.group_size
     if d % 2 or d % g:
         raise ValueError("d must be even and a multiple of the group size")
@@ -107,6 +154,38 @@ def make_head(shape: HeadShape, seed: int = 0) -> Dict[str, np.ndarray]:
         "res_scales": _fp16_scales(s["res_scales"], base_r, (V, d // g)),
         "core_u": _int8_codes(s["core_u"], (V, rc)),
         "core_u_scale": _fp16_scales(s["core_u_scale"], base_c, (rc,)),
+        "core_v": _int8_codes(s["core_v"], (d, rc)),
+        "core_v_scale": _fp16_scales(s["core_v_scale"], base_c, (rc,)),
+        "corr_a": _int8_codes(s["corr_a"], (V, rr)),
+        "corr_a_scale": _fp16_scales(s["corr_a_scale"], base_w, (V,)),
+        "corr_b": _int8_codes(s["corr_b"], (d, rr)),
+        "corr_b_scale": _fp16_scales(s["corr_b_scale"], base_w, (d // g, rr)),
+    }
+    return {k: np.ascontiguousarray(v) for k, v in head.items()}
+
+
+_HEAD_STREAMS_SC4 = (
+    "res_codes", "res_scale_codes", "res_row_scale", "core_u5", "core_u_scale", "core_v", "core_v_scale",
+    "corr_a", "corr_a_scale", "corr_b", "corr_b_scale",
+)
+
+
+def _make_head_sc4(shape: HeadShape, seed: int) -> Dict[str, np.ndarray]:
+    """The paper's packed format ("sc4" above), same element rms targets."""
+    V, d, rc, rr, g = shape.V, shape.d, shape.core_rank, shape.corr_rank, shape.group_size
+    if d % 2 or d % g:
+        raise ValueError("d must be even and a multiple of the group size")
+    s = _streams(seed, _HEAD_STREAMS_SC4)
+    base_r = _RMS_RESIDUAL / _RMS_INT4 / _RMS_SCALE_MULT
+    base_c = float(np.sqrt(_RMS_CORE / (np.sqrt(max(rc, 1)) * _MS_INT8)))
+    base_w = float(np.sqrt(_RMS_CORRECTION / (np.sqrt(max(rr, 1)) * _MS_INT8)))
+    G = d // g
+    head = {
+        "res_codes": s["res_codes"].integers(0, 256, size=(V, d // 2), dtype=np.uint8),
+        "res_scale_codes": _uniform_bits(s["res_scale_codes"], V, shape.scale_code_bytes, 4 * G),
+        "res_row_scale": _fp16_scales(s["res_row_scale"], base_r, (V,)),
+        "core_u5": _uniform_bits(s["core_u5"], V, shape.core_u5_bytes, 5 * rc),
+        "core_u_scale": _fp16_scales(s["core_u_scale"], base_c * np.sqrt(_MS_INT8 / _MS_INT5), (rc,)),
         "core_v": _int8_codes(s["core_v"], (d, rc)),
         "core_v_scale": _fp16_scales(s["core_v_scale"], base_c, (rc,)),
         "corr_a": _int8_codes(s["corr_a"], (V, rr)),

@@ -7,7 +7,10 @@ Each check raises AssertionError when the oracle disagrees with:
     U V^T; zero ranks = plain group-wise INT4 matmul);
   - closed forms of the cross entropy (uniform logits give log V);
   - a pure-Python brute force of Eqs. 3, 6 and 7 on tiny heads;
-  - the paper's printed dense-head sizes (Section 3.3, Table 1);
+  - the paper's printed dense-head sizes and its packed Qwen head size
+    (Section 3.3, Table 1);
+  - for the paper's own format (5-bit core codes, quantised group scales):
+    numpy's bit unpacking, a brute force, and the equal int8-format head;
   - invariants (linearity in x, vocabulary permutation, argmax tie rule).
 
 The same checks run against deliberately mutated builds of the oracle in
@@ -251,8 +254,170 @@ def check_packed_bytes(oracle):
         assert oracle.packed_bytes(shape) == counted, shape
 
 
+# ---------------------------------------------------------------------------
+# The paper's packed format ("sc4": 5-bit core left factor, 4-bit group-scale
+# codes times an fp16 row scale).
+# ---------------------------------------------------------------------------
+PIN_SHAPE_SC4 = HeadShape(V=24, d=80, core_rank=5, corr_rank=3, group_size=16, fmt="sc4")  # 5 groups: odd
+
+
+def _np_int5(packed: np.ndarray, rank: int) -> np.ndarray:
+    """5-bit two's complement fields, LSB first, through numpy's unpackbits."""
+    bits = np.unpackbits(packed, axis=1, bitorder="little")[:, :5 * rank].reshape(packed.shape[0], rank, 5)
+    v = (bits.astype(np.int64) << np.arange(5)).sum(axis=2)
+    return np.where(v >= 16, v - 32, v)
+
+
+def _np_scale_codes(packed: np.ndarray, groups: int) -> np.ndarray:
+    q = np.empty((packed.shape[0], 2 * packed.shape[1]), dtype=np.int64)
+    q[:, 0::2] = packed & 0xF
+    q[:, 1::2] = packed >> 4
+    return q[:, :groups]
+
+
+def check_int5_unpack(oracle):
+    # Written out by hand: codes (1, -1, -16) are the bit string
+    # 10000 11111 00001 (LSB first), i.e. bytes 0xE1, 0x43.
+    assert oracle.unpack_int5(np.array([[0xE1, 0x43]], dtype=np.uint8), 3).tolist() == [[1, -1, -16]]
+    # (15, 0, 7, -8): bits 0-3, 10-12, 18-19 set -> 0x0F, 0x1C, 0x0C (padding bits zero).
+    assert oracle.unpack_int5(np.array([[0x0F, 0x1C, 0x0C]], dtype=np.uint8), 4).tolist() == [[15, 0, 7, -8]]
+    # Every code value at every bit offset (j = 0..7 covers offsets 0, 5, 2, 7, 4, 1, 6, 3).
+    codes = np.array([[(v + 7 * j) % 32 - 16 for j in range(8)] for v in range(32)], dtype=np.int64)
+    bits = ((codes[:, :, None] & 31) >> np.arange(5)) & 1
+    packed = np.packbits(bits.reshape(32, 40).astype(np.uint8), axis=1, bitorder="little")
+    assert np.array_equal(oracle.unpack_int5(packed, 8), codes)
+    # Random rows of several ranks against numpy's bit unpacking.
+    rng = np.random.default_rng(21)
+    for rank in (1, 3, 10, 13):
+        nb = (5 * rank + 7) // 8
+        raw = rng.integers(0, 256, size=(9, nb), dtype=np.uint8)
+        assert np.array_equal(oracle.unpack_int5(raw, rank), _np_int5(raw, rank)), rank
+
+
+def check_scale_code_unpack(oracle):
+    assert oracle.unpack_scale_codes(np.array([[0x5A, 0xF0]], dtype=np.uint8), 4).tolist() == [[10, 5, 0, 15]]
+    assert oracle.unpack_scale_codes(np.array([[0x31, 0x07]], dtype=np.uint8), 3).tolist() == [[1, 3, 7]]
+    raw = np.random.default_rng(22).integers(0, 256, size=(7, 5), dtype=np.uint8)
+    assert np.array_equal(oracle.unpack_scale_codes(raw, 9), _np_scale_codes(raw, 9))
+
+
+def _dq_sc4(head, shape):
+    """Components of an sc4 head decoded with numpy (not the oracle)."""
+    g = shape.group_size
+    codes = np.empty((shape.V, shape.d), dtype=np.int64)
+    b = head["res_codes"].astype(np.int64)
+    codes[:, 0::2] = ((b & 0xF) ^ 0x8) - 0x8
+    codes[:, 1::2] = (((b >> 4) & 0xF) ^ 0x8) - 0x8
+    f16 = lambda a: a.view(np.float16).astype(np.float64)  # noqa: E731
+    s = f16(head["res_row_scale"])[:, None] * (_np_scale_codes(head["res_scale_codes"], shape.groups) + 1)
+    res = codes * np.repeat(s, g, axis=1)
+    U = _np_int5(head["core_u5"], shape.core_rank) * f16(head["core_u_scale"])[None, :]
+    Vc = head["core_v"].astype(np.float64) * f16(head["core_v_scale"])[None, :]
+    A = head["corr_a"].astype(np.float64) * f16(head["corr_a_scale"])[:, None]
+    B = head["corr_b"].astype(np.float64) * np.repeat(f16(head["corr_b_scale"]), g, axis=0)
+    return res, U, Vc, A, B
+
+
+def check_sc4_components(oracle, shape=PIN_SHAPE_SC4):
+    head = make_head(shape, seed=23)
+    res, U, Vc, A, B = _dq_sc4(head, shape)
+    for name, ref in (("residual", res), ("core_u", U), ("core_v", Vc), ("corr_a", A), ("corr_b", B)):
+        got = oracle.component(head, shape, name)
+        assert np.array_equal(got, ref), f"sc4 component {name} is not exactly code * scale"
+    W = oracle.dequant_rows(head, shape)
+    assert np.allclose(W, res + U @ Vc.T + A @ B.T, rtol=1e-13, atol=1e-15)
+
+
+def _brute_force_logits_sc4(head, shape, x_bits):
+    """Pure-Python loops with per-element bit decoding of the sc4 fields."""
+    V, d, g, rc, rr = shape.V, shape.d, shape.group_size, shape.core_rank, shape.corr_rank
+    nb_u = (5 * rc + 7) // 8
+
+    def u5(n, j):
+        row = [int(v) for v in head["core_u5"][n, :nb_u]]
+        word = sum(v << (8 * i) for i, v in enumerate(row))
+        c = (word >> (5 * j)) & 31
+        return c - 32 if c >= 16 else c
+
+    def scale(n, grp):
+        byte = int(head["res_scale_codes"][n, grp // 2])
+        q = (byte >> 4) if grp % 2 else (byte & 15)
+        return _f16(head["res_row_scale"][n]) * (q + 1)
+
+    y = [[0.0] * V for _ in range(x_bits.shape[0])]
+    for n in range(V):
+        w = []
+        for k in range(d):
+            v = _int4_from_byte(int(head["res_codes"][n, k // 2]), high=(k % 2 == 1)) * scale(n, k // g)
+            for j in range(rc):
+                v += (u5(n, j) * _f16(head["core_u_scale"][j])) * (
+                    int(head["core_v"][k, j]) * _f16(head["core_v_scale"][j]))
+            for j in range(rr):
+                v += (int(head["corr_a"][n, j]) * _f16(head["corr_a_scale"][n])) * (
+                    int(head["corr_b"][k, j]) * _f16(head["corr_b_scale"][k // g, j]))
+            w.append(v)
+        for m in range(x_bits.shape[0]):
+            y[m][n] = math.fsum(_bf16(x_bits[m, k]) * w[k] for k in range(d))
+    return np.array(y)
+
+
+def check_sc4_brute_force(oracle, shape=PIN_SHAPE_SC4):
+    head = make_head(shape, seed=24)
+    x = make_hidden(shape.d, 2, seed=24)
+    ref = _brute_force_logits_sc4(head, shape, x)
+    got = oracle.logits(head, shape, x)
+    assert np.allclose(got, ref, rtol=1e-12, atol=1e-12 * np.abs(ref).max()), "sc4 logits differ from brute force"
+
+
+def check_sc4_equals_int8_form(oracle):
+    """An sc4 head whose group scales s_row (q + 1) are exact in fp16 is the
+    same head as the int8-format head holding those scales and the widened
+    5-bit codes: the two must give identical logits."""
+    shape = HeadShape(V=33, d=128, core_rank=7, corr_rank=4, group_size=32, fmt="sc4")
+    head = make_head(shape, seed=25)
+    rng = np.random.default_rng(25)
+    # Row scales 2^-12 (1 + k/64): 7 significant bits, so s_row * (q + 1) <= 16 s_row fits fp16 exactly.
+    s_row = (2.0 ** -12) * (1 + rng.integers(0, 64, size=shape.V) / 64.0)
+    head["res_row_scale"] = s_row.astype(np.float16).view(np.uint16)
+    q = _np_scale_codes(head["res_scale_codes"], shape.groups)
+    scales = (s_row[:, None] * (q + 1)).astype(np.float16)
+    assert np.array_equal(scales.astype(np.float64), s_row[:, None] * (q + 1))
+    i8shape = HeadShape(V=shape.V, d=shape.d, core_rank=shape.core_rank, corr_rank=shape.corr_rank,
+                        group_size=shape.group_size)
+    i8 = {k: v for k, v in head.items() if k not in ("res_scale_codes", "res_row_scale", "core_u5")}
+    i8["res_scales"] = np.ascontiguousarray(scales.view(np.uint16))
+    i8["core_u"] = np.ascontiguousarray(_np_int5(head["core_u5"], shape.core_rank).astype(np.int8))
+    x = make_hidden(shape.d, 3, seed=25)
+    assert np.array_equal(oracle.logits(head, shape, x), oracle.logits(i8, i8shape, x))
+
+
+def check_paper_packed_storage(oracle):
+    """Eq. 10 over the sc4 format reproduces the paper's packed size of the
+    Qwen3-8B head (Table 1) within 0.1 MiB (0.03 %) and its compression."""
+    rows = []
+    with open(os.path.join(GOLDEN, "paper_table1_packed_qwen_mib.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                name, V, D, rc, rr, g, mb, ratio = line.split()
+                rows.append((name, int(V), int(D), int(rc), int(rr), int(g), float(mb), float(ratio)))
+    assert len(rows) == 1
+    for name, V, D, rc, rr, g, mb, ratio in rows:
+        shape = HeadShape(V=V, d=D, core_rank=rc, corr_rank=rr, group_size=g, fmt="sc4")
+        got = oracle.packed_bytes(shape)
+        assert abs(got / 2**20 - mb) < 0.1, (name, got / 2**20)
+        assert abs(oracle.dense_bf16_bytes(V, D) / got - ratio) < 0.002, name
+        # The format's own arrays count to the same bytes (small head, same rule).
+    for shape in (PIN_SHAPE_SC4, HeadShape(V=50, d=192, core_rank=10, corr_rank=6, group_size=64, fmt="sc4"),
+                  HeadShape(V=7, d=96, core_rank=0, corr_rank=0, group_size=32, fmt="sc4")):
+        head = make_head(shape, seed=26)
+        counted = sum(a.nbytes for k, a in head.items() if not (k == "corr_a_scale" and shape.corr_rank == 0))
+        assert oracle.packed_bytes(shape) == counted, shape
+
+
 ALL_CHECKS = [
     check_int4_unpack, check_fp16_decode, check_bf16_decode, check_core_only, check_group_int4,
     check_components, check_brute_force, check_cross_entropy, check_invariants,
     check_paper_dense_sizes, check_packed_bytes,
+    check_int5_unpack, check_scale_code_unpack, check_sc4_components, check_sc4_brute_force,
+    check_sc4_equals_int8_form, check_paper_packed_storage,
 ]

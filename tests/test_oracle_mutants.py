@@ -21,8 +21,10 @@ MUTANTS = {
     "int4_nibble_order": ("int nib = (k % 2 == 0) ? (byte & 0x0F)", "int nib = (k % 2 == 1) ? (byte & 0x0F)"),
     "fp16_exponent_bias": ("v = ldexp((double)(1024 + f), e - 25);", "v = ldexp((double)(1024 + f), e - 24);"),
     "bf16_exponent_bias": ("v = ldexp((double)(128 + f), e - 134);", "v = ldexp((double)(128 + f), e - 135);"),
-    "residual_scale_group": ("double s_r = oracle_fp16_value(h->res_scales[n * G + k / g]);",
-                             "double s_r = oracle_fp16_value(h->res_scales[n * G + (k / g + 1) % G]);"),
+    "residual_scale_group": ("double s_r = res_scale(h, n, k / g);",
+                             "double s_r = res_scale(h, n, (k / g + 1) % (d / g));"),
+    "int8_residual_scale_row": ("return oracle_fp16_value(h->res_scales[n * G + grp]);",
+                                "return oracle_fp16_value(h->res_scales[((n + 1) % h->V) * G + grp]);"),
     "core_scale_swapped": ("c->su[j] = oracle_fp16_value(h->core_u_scale[j]);",
                            "c->su[j] = oracle_fp16_value(h->core_v_scale[j]);"),
     "core_right_transposed": ("c->vdq[k * rc + j] = (double)h->core_v[k * rc + j]",
@@ -37,7 +39,19 @@ MUTANTS = {
     "lse_not_shifted": ("s += exp(row[n] - mx);", "s += exp(row[n]);"),
     "ce_wrong_logit": ("ce[m] = lse - row[t];", "ce[m] = lse - row[arg];"),
     "argmax_tie_high": ("if (row[n] > mx) { mx = row[n]; arg = n; }", "if (row[n] >= mx) { mx = row[n]; arg = n; }"),
-    "bytes_scale_dropped": ("bytes += G * rr * 2;", "bytes += 0;"),
+    "bytes_scale_dropped": ("bytes += G * rr * 2;     /* correction group scales */", "bytes += 0;"),
+    # the paper's packed format (5-bit core codes, 4-bit group-scale codes)
+    "int5_sign_extension": ("return v >= 16 ? v - 32 : v;", "return v >= 16 ? v - 31 : v;"),
+    "int5_bit_order": ("v |= ((row[bit / 8] >> (bit % 8)) & 1) << b;", "v |= ((row[bit / 8] >> (bit % 8)) & 1) << (4 - b);"),
+    "int5_row_stride": ("h->core_u5 + n * ((5 * (int64_t)h->core_rank + 7) / 8)",
+                        "h->core_u5 + n * ((5 * (int64_t)h->core_rank) / 8)"),
+    "scale_code_offset_dropped": ("scale_code(h->res_scale_codes + n * nb, grp) + 1);",
+                                  "scale_code(h->res_scale_codes + n * nb, grp) + 0);"),
+    "scale_code_nibble_order": ("return (grp % 2 == 0) ? (byte & 0x0F)", "return (grp % 2 == 1) ? (byte & 0x0F)"),
+    "scale_code_row_stride": ("const int64_t nb = (G + 1) / 2;\n    return", "const int64_t nb = G / 2;\n    return"),
+    "row_scale_index": ("oracle_fp16_value(h->res_row_scale[n])", "oracle_fp16_value(h->res_row_scale[(n + 1) % h->V])"),
+    "sc4_bytes_row_scales_dropped": ("bytes += V * 2;                /* residual row scales", "bytes += 0;  /*"),
+    "sc4_bytes_core_unpacked": ("bytes += V * ((5 * rc + 7) / 8);", "bytes += V * rc;"),
 }
 
 
