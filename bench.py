@@ -41,6 +41,9 @@ WORKLOADS = {
     "qwen3-8b-decode": ("qwen3-8b", 1, "logits"),
     "qwen3-8b-prefill": ("qwen3-8b", 4096, "logits"),
     "qwen3-8b-prefill-ce": ("qwen3-8b", 4096, "ce"),
+    # the same head shape in the paper's own packed format (r_c = 10, r_r = 6, g = 64)
+    "qwen3-8b-sc4-decode": ("qwen3-8b-sc4", 1, "logits"),
+    "qwen3-8b-sc4-prefill": ("qwen3-8b-sc4", 4096, "logits"),
     "gemma-4-e4b-decode": ("gemma-4-e4b", 1, "logits"),
     "gemma-4-e4b-prefill": ("gemma-4-e4b", 2048, "logits"),
     "tiny": ("tiny", 4, "logits"),
@@ -93,9 +96,16 @@ def load_peaks():
 # Algorithmic work (what the method must move or compute per call).
 # ---------------------------------------------------------------------------
 def packed_vocab_bytes(shape) -> int:
-    """Bytes of the V-indexed packed components the streaming kernel reads."""
+    """Bytes of the V-indexed packed components the streaming kernel reads
+    (in the paper's packed format: 4-bit group-scale codes, fp16 row scales
+    and 5-bit core left codes in place of fp16 group scales and INT8 codes)."""
     V, d, rc, rr, g = shape.V, shape.d, shape.core_rank, shape.corr_rank, shape.group_size
-    return V * d // 2 + V * (d // g) * 2 + V * rc + V * rr + (V * 2 if rr else 0)
+    G = d // g
+    if getattr(shape, "fmt", "int8") == "sc4":
+        scales, core = V * ((G + 1) // 2) + V * 2, V * ((5 * rc + 7) // 8)
+    else:
+        scales, core = V * G * 2, V * rc
+    return V * d // 2 + scales + core + V * rr + (V * 2 if rr else 0)
 
 
 def packed_bytes(shape) -> int:
@@ -365,7 +375,8 @@ def run_ours(args, rank, world, local_rank):
         "config": {"workload": f"{shape_name} head, {'decode' if M <= 16 else 'prefill'} M={M}, "
                                f"{'logits bf16' if mode == 'logits' else 'fused CE'}",
                    "V": shape.V, "d": shape.d, "core_rank": shape.core_rank, "corr_rank": shape.corr_rank,
-                   "group_size": shape.group_size, "M": M, "parallelism": f"replicas x{world}",
+                   "group_size": shape.group_size, "format": shape.fmt, "M": M,
+                   "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2: the packed head (%.1f MB) exceeds the 129 MB L2, so every "
                          "forward streams it from HBM" % (packed_bytes(shape) / 1e6)},
         "roofline": roof,
@@ -382,20 +393,37 @@ def run_ours(args, rank, world, local_rank):
         result["decode_sweep"] = decode_sweep(pack, shape, peaks, world, local_rank)
         result["prefill"] = prefill_block(pack, shape, peaks, world, local_rank)
         result["dense_bf16_cublas"] = dense_comparator(shape, world, local_rank)
+        result["crossover"] = crossover_sweep(pack, shape, world, local_rank)
     pack.close()
+    if not args.no_extras and args.workload == "qwen3-8b-decode":
+        result["sc4"] = sc4_block(peaks, world, local_rank)
     if rank == 0 and not args.no_cpu_baseline and world == 1:
         result["cpu_baseline"] = cpu_baseline(wl, x_np, M, budget_s=args.cpu_budget)
     return result
 
 
-def decode_sweep(pack, shape, peaks, world, local_rank):
+def sc4_block(peaks, world, local_rank):
+    """The Qwen3-8B head in the paper's own packed format (5-bit core left
+    codes, 4-bit group-scale codes, r_c = 10, r_r = 6, g = 64): decode and
+    prefill on the same footing as the lines above."""
+    wl = Workload("qwen3-8b-sc4")
+    pack = wl.open()
+    res = {"workload": "qwen3-8b-sc4 head (V=151936, d=4096, r_c=10, r_r=6, g=64, paper's packed format)",
+           "packed_bytes": packed_bytes(wl.shape),
+           "decode_sweep": decode_sweep(pack, wl.shape, peaks, world, local_rank, Ms=(1, 4, 8, 16)),
+           "prefill": prefill_block(pack, wl.shape, peaks, world, local_rank)}
+    pack.close()
+    return res
+
+
+def decode_sweep(pack, shape, peaks, world, local_rank, Ms=(1, 2, 4, 8, 16)):
     import torch
 
     from paper_2608_02703_gb300 import archead
     from synth import make_hidden
 
     out = []
-    for M in (1, 2, 4, 8, 16):
+    for M in Ms:
         x = torch.from_numpy(make_hidden(shape.d, M, seed=2, n_outliers=shape.n_outliers).view(np.int16)).cuda()
         y = torch.empty((M, shape.V), dtype=torch.bfloat16, device="cuda")
         fn = lambda: archead.archead_forward(pack, x, M, y, archead.OUT_BF16)  # noqa: E731
@@ -432,6 +460,44 @@ def prefill_block(pack, shape, peaks, world, local_rank):
     st = archead.archead_sync_status(pack)
     res["status"] = archead.archead_status_string(st)
     return res
+
+
+def crossover_sweep(pack, shape, world, local_rank):
+    """Batch sweep on one head: per M the decode kernel (tokens 16 at a time),
+    the prefill kernel, the automatic choice and a dense BF16 cuBLAS GEMM of
+    the same shape, each as microseconds per call (bf16 logits out)."""
+    import torch
+
+    from paper_2608_02703_gb300 import archead
+    from synth import make_hidden
+
+    g = torch.Generator(device="cuda")
+    g.manual_seed(0)
+    W = (torch.randn((shape.V, shape.d), generator=g, device="cuda", dtype=torch.float32) * 0.01).to(torch.bfloat16)
+    dev = torch.device("cuda", local_rank)
+    rows = []
+    for M in (1, 4, 16, 64, 256, 1024, 4096, 8192):
+        x = torch.from_numpy(make_hidden(shape.d, M, seed=5, n_outliers=shape.n_outliers).view(np.int16)).cuda()
+        y = torch.empty((M, shape.V), dtype=torch.bfloat16, device="cuda")
+        k = 200 if M <= 16 else (20 if M <= 1024 else 4)
+        row = {"M": M}
+        for name, path in (("decode_us", archead.PATH_DECODE), ("prefill_us", archead.PATH_PREFILL),
+                           ("auto_us", archead.PATH_AUTO)):
+            fn = lambda: archead.archead_forward_path(pack, x, M, y, archead.OUT_BF16, path)  # noqa: E731
+            kk = max(2, k // 8) if (path == archead.PATH_DECODE and M >= 1024) else k
+            secs = max_over_ranks(timed_loop(fn, kk, 3, world), world, dev)
+            row[name] = round(secs / kk * 1e6, 2)
+        xb = x.view(torch.bfloat16)
+        fn = lambda: torch.matmul(xb, W.t())  # noqa: E731
+        secs = max_over_ranks(timed_loop(fn, k, 3, world), world, dev)
+        row["dense_bf16_us"] = round(secs / k * 1e6, 2)
+        row["auto_tokens_s"] = round(world * M / (row["auto_us"] / 1e6), 1)
+        rows.append(row)
+        del y
+    st = archead.archead_sync_status(pack)
+    del W
+    torch.cuda.empty_cache()
+    return {"rows": rows, "status": archead.archead_status_string(st)}
 
 
 def dense_comparator(shape, world, local_rank):

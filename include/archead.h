@@ -63,6 +63,12 @@ typedef enum {
   ARCHEAD_OUT_FP32 = 1  /* logits as the fp32 accumulators                               */
 } archead_out_dtype;
 
+/* Stored format of the packed head (archead_desc.format). */
+typedef enum {
+  ARCHEAD_FORMAT_INT8 = 0, /* INT8 core left factor, one fp16 scale per residual group          */
+  ARCHEAD_FORMAT_SC4 = 1   /* the paper's format: 5-bit core left factor, 4-bit scale codes    */
+} archead_format;
+
 typedef enum {
   ARCHEAD_PATH_AUTO = 0,    /* decode kernel for M <= 16, prefill kernel above          */
   ARCHEAD_PATH_DECODE = 1,  /* memory-bound decode kernel (tokens taken 16 at a time)   */
@@ -92,6 +98,20 @@ typedef enum {
  * A rank of 0 drops that branch (its pointers may then be NULL): r_c = r_r = 0
  * is the plain group-wise INT4 head, r_r = 0 the "core only" variant.
  *
+ * format = ARCHEAD_FORMAT_SC4 selects the paper's own packed format
+ * (Section 3.2, Eq. 3: Q_5 core left factor and the SC4 residual with
+ * quantised group scales; Appendix C).  Three fields change meaning:
+ *   res_scales    uint8 [V][ceil(G/2)]  4-bit unsigned group-scale codes q,
+ *                                 low nibble = even group, G = d/g;
+ *   res_row_scale fp16  [V]       one per row; the group scale is
+ *                                 s_R[n, grp] = res_row_scale[n] * (q + 1);
+ *   core_u        uint8 [V][ceil(5 r_c / 8)]  5-bit two's complement codes
+ *                                 (-16..15), code j in bits 5j..5j+4 of the
+ *                                 row's bytes read as one little-endian bit
+ *                                 string (unused top bits ignored).
+ * Everything else is as above.  res_row_scale is read only in this format
+ * (callers of the INT8 format may pass a shorter struct without it).
+ *
  * Supported envelope: V >= 1; d a multiple of 64 and of g; g in {32, 64,
  * 128, 256}; 0 <= r_c, r_r <= 256.
  */
@@ -101,7 +121,7 @@ typedef struct {
   int32_t core_rank;   /* r_c */
   int32_t corr_rank;   /* r_r */
   int32_t group_size;  /* g */
-  int32_t reserved;    /* must be 0 */
+  int32_t format;      /* archead_format */
   const void *res_codes;
   const void *res_scales;
   const void *core_u;
@@ -112,6 +132,7 @@ typedef struct {
   const void *corr_a_scale;
   const void *corr_b;
   const void *corr_b_scale;
+  const void *res_row_scale; /* ARCHEAD_FORMAT_SC4 only */
 } archead_desc;
 
 /*
@@ -182,8 +203,8 @@ ARCHEAD_API archead_status archead_forward_host(archead_pack *pack, const void *
 
 /*
  * Persistent storage of the packed head (paper, Section 3.3, Eq. 10): the
- * sum of numel * element_size over the stored components listed above.  The
- * correction's row scales count only when r_r > 0.
+ * sum of numel * element_size over the stored components listed above, in
+ * the pack's format.  The correction's row scales count only when r_r > 0.
  */
 ARCHEAD_API int64_t archead_pack_bytes(const archead_pack *pack);
 

@@ -28,6 +28,9 @@ ERR_TARGET_RANGE = 6
 OUT_BF16 = 0
 OUT_FP32 = 1
 
+FORMAT_INT8 = 0
+FORMAT_SC4 = 1
+
 PATH_AUTO = 0
 PATH_DECODE = 1
 PATH_PREFILL = 2
@@ -57,12 +60,13 @@ class archead_desc(ctypes.Structure):  # noqa: N801 - mirrors the C struct name
     _fields_ = [
         ("vocab", ctypes.c_int64), ("hidden", ctypes.c_int64),
         ("core_rank", ctypes.c_int32), ("corr_rank", ctypes.c_int32),
-        ("group_size", ctypes.c_int32), ("reserved", ctypes.c_int32),
+        ("group_size", ctypes.c_int32), ("format", ctypes.c_int32),
         ("res_codes", ctypes.c_void_p), ("res_scales", ctypes.c_void_p),
         ("core_u", ctypes.c_void_p), ("core_u_scale", ctypes.c_void_p),
         ("core_v", ctypes.c_void_p), ("core_v_scale", ctypes.c_void_p),
         ("corr_a", ctypes.c_void_p), ("corr_a_scale", ctypes.c_void_p),
         ("corr_b", ctypes.c_void_p), ("corr_b_scale", ctypes.c_void_p),
+        ("res_row_scale", ctypes.c_void_p),
     ]
 
 
@@ -165,12 +169,19 @@ class Pack:
 
 
 def archead_pack_create(head: Dict, shape, stream=None) -> Pack:
-    """Build a pack from canonical arrays (numpy host arrays or torch tensors)."""
+    """Build a pack from canonical arrays (numpy host arrays or torch tensors).
+
+    The INT8 format takes the arrays named as the struct fields; the paper's
+    format (shape.fmt == "sc4") takes res_scale_codes, res_row_scale and
+    core_u5 in place of res_scales and core_u."""
+    sc4 = getattr(shape, "fmt", "int8") == "sc4"
     d = archead_desc(vocab=shape.V, hidden=shape.d, core_rank=shape.core_rank, corr_rank=shape.corr_rank,
-                     group_size=shape.group_size, reserved=0)
+                     group_size=shape.group_size, format=FORMAT_SC4 if sc4 else FORMAT_INT8)
+    source = {"res_scales": "res_scale_codes", "core_u": "core_u5"} if sc4 else {"res_row_scale": None}
     keep = []
     for name, _ in archead_desc._fields_[6:]:
-        a = head.get(name)
+        key = source.get(name, name)
+        a = head.get(key) if key is not None else None
         if a is not None and hasattr(a, "flags") and not a.flags["C_CONTIGUOUS"]:
             a = np.ascontiguousarray(a)
         if a is not None and hasattr(a, "is_contiguous") and not a.is_contiguous():

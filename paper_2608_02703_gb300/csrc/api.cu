@@ -41,8 +41,9 @@ cudaError_t dev_alloc(archead_pack *p, T **ptr, size_t bytes) {
 
 void free_pack(archead_pack *p) {
   if (!p) return;
-  void *bufs[] = {p->codes, p->scales, p->lr_codes, p->s_a,    p->q_v,    p->q_b,   p->lr_t, p->s_u,
-                  p->s_v,   p->s_b,    p->err,      p->ws,     p->xh_dev, p->yh_dev, p->counters};
+  void *bufs[] = {p->codes, p->scales, p->scodes, p->s_row,  p->lr_codes, p->s_a,    p->q_v,
+                  p->q_b,   p->lr_t,   p->s_u,    p->s_v,    p->s_b,      p->err,    p->ws,
+                  p->xh_dev, p->yh_dev, p->counters};
   for (void *b : bufs)
     if (b) cudaFree(b);
   for (auto &t : p->timers)
@@ -175,6 +176,10 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   DecodeParams dp{};
   dp.codes = p->codes;
   dp.scales = p->scales;
+  dp.scodes = p->scodes;
+  dp.s_row = p->s_row;
+  dp.sc4 = p->sc4;
+  dp.G_pad2 = p->G_pad2;
   dp.lr_codes = p->lr_codes;
   dp.s_a = p->s_a;
   dp.x = static_cast<const uint16_t *>(x);
@@ -314,11 +319,15 @@ archead_status archead_pack_create(const archead_desc *desc, void *stream, arche
   if (!desc) return ARCHEAD_ERR_INVALID_ARG;
   const int64_t V = desc->vocab, d = desc->hidden;
   const int rc = desc->core_rank, rr = desc->corr_rank, g = desc->group_size;
-  if (V < 1 || d < 64 || d % 64 != 0 || desc->reserved != 0) return ARCHEAD_ERR_INVALID_ARG;
+  const int fmt = desc->format;
+  if (fmt != ARCHEAD_FORMAT_INT8 && fmt != ARCHEAD_FORMAT_SC4) return ARCHEAD_ERR_INVALID_ARG;
+  const bool sc4 = fmt == ARCHEAD_FORMAT_SC4;
+  if (V < 1 || d < 64 || d % 64 != 0) return ARCHEAD_ERR_INVALID_ARG;
   if (!(g == 32 || g == 64 || g == 128 || g == 256) || d % g != 0) return ARCHEAD_ERR_INVALID_ARG;
   if (rc < 0 || rr < 0 || rc > 256 || rr > 256) return ARCHEAD_ERR_INVALID_ARG;
   if (d > (1 << 20) || V > ((int64_t)1 << 31) - 256) return ARCHEAD_ERR_UNSUPPORTED;
   if (!desc->res_codes || !desc->res_scales) return ARCHEAD_ERR_INVALID_ARG;
+  if (sc4 && !desc->res_row_scale) return ARCHEAD_ERR_INVALID_ARG;
   if (rc > 0 && (!desc->core_u || !desc->core_u_scale || !desc->core_v || !desc->core_v_scale))
     return ARCHEAD_ERR_INVALID_ARG;
   if (rr > 0 && (!desc->corr_a || !desc->corr_a_scale || !desc->corr_b || !desc->corr_b_scale))
@@ -344,6 +353,8 @@ archead_status archead_pack_create(const archead_desc *desc, void *stream, arche
   p->G = (int)(d / g);
   p->d_pad = (int)round_up(d, 128);
   p->G_pad = p->d_pad / g;
+  p->sc4 = sc4 ? 1 : 0;
+  p->G_pad2 = (p->G_pad + 1) / 2;
   p->num_tiles = (int)((V + kTileRows - 1) / kTileRows);
   p->V_pad = (int64_t)p->num_tiles * kTileRows;
   p->rcp = (int)round_up(rc, 32);
@@ -354,7 +365,12 @@ archead_status archead_pack_create(const archead_desc *desc, void *stream, arche
 
   const size_t G = p->G;
   if ((e = dev_alloc(p, &p->codes, (size_t)p->V_pad * p->d_pad / 2)) != cudaSuccess) return fail(e);
-  if ((e = dev_alloc(p, &p->scales, (size_t)p->V_pad * p->G_pad * 2)) != cudaSuccess) return fail(e);
+  if (sc4) {
+    if ((e = dev_alloc(p, &p->scodes, (size_t)p->V_pad * p->G_pad2)) != cudaSuccess) return fail(e);
+    if ((e = dev_alloc(p, &p->s_row, (size_t)p->V_pad * 2)) != cudaSuccess) return fail(e);
+  } else {
+    if ((e = dev_alloc(p, &p->scales, (size_t)p->V_pad * p->G_pad * 2)) != cudaSuccess) return fail(e);
+  }
   if ((e = dev_alloc(p, &p->lr_codes, (size_t)p->num_tiles * p->nls * kLrStepBytes)) != cudaSuccess) return fail(e);
   if ((e = dev_alloc(p, &p->s_a, (size_t)p->V_pad * 2)) != cudaSuccess) return fail(e);
   if ((e = dev_alloc(p, &p->q_v, (size_t)d * rc)) != cudaSuccess) return fail(e);
@@ -368,9 +384,10 @@ archead_status archead_pack_create(const archead_desc *desc, void *stream, arche
 
   // Canonical components: the V-indexed ones pass through temporaries on the
   // device and are re-tiled; the d-indexed ones are copied as they are.
-  uint8_t *t_codes = nullptr, *t_scales = nullptr, *t_u = nullptr, *t_a = nullptr, *t_sa = nullptr;
+  uint8_t *t_codes = nullptr, *t_scales = nullptr, *t_u = nullptr, *t_a = nullptr, *t_sa = nullptr,
+          *t_srow = nullptr;
   auto free_tmp = [&]() {
-    for (void *b : {(void *)t_codes, (void *)t_scales, (void *)t_u, (void *)t_a, (void *)t_sa})
+    for (void *b : {(void *)t_codes, (void *)t_scales, (void *)t_u, (void *)t_a, (void *)t_sa, (void *)t_srow})
       if (b) cudaFree(b);
   };
   auto tmp_copy = [&](uint8_t **dst, const void *src, size_t bytes) -> cudaError_t {
@@ -380,8 +397,10 @@ archead_status archead_pack_create(const archead_desc *desc, void *stream, arche
     return cudaMemcpyAsync(*dst, src, bytes, cudaMemcpyDefault, s);
   };
   e = tmp_copy(&t_codes, desc->res_codes, (size_t)V * d / 2);
-  if (e == cudaSuccess) e = tmp_copy(&t_scales, desc->res_scales, (size_t)V * G * 2);
-  if (e == cudaSuccess && rc > 0) e = tmp_copy(&t_u, desc->core_u, (size_t)V * rc);
+  // SC4: 4-bit scale codes (ceil(G/2) bytes a row), fp16 row scales, 5-bit core codes (ceil(5 r_c/8) bytes a row).
+  if (e == cudaSuccess) e = tmp_copy(&t_scales, desc->res_scales, sc4 ? (size_t)V * ((G + 1) / 2) : (size_t)V * G * 2);
+  if (e == cudaSuccess && sc4) e = tmp_copy(&t_srow, desc->res_row_scale, (size_t)V * 2);
+  if (e == cudaSuccess && rc > 0) e = tmp_copy(&t_u, desc->core_u, sc4 ? (size_t)V * ((5 * rc + 7) / 8) : (size_t)V * rc);
   if (e == cudaSuccess && rr > 0) e = tmp_copy(&t_a, desc->corr_a, (size_t)V * rr);
   if (e == cudaSuccess && rr > 0) e = tmp_copy(&t_sa, desc->corr_a_scale, (size_t)V * 2);
   if (e == cudaSuccess && rc > 0) e = cudaMemcpyAsync(p->q_v, desc->core_v, (size_t)d * rc, cudaMemcpyDefault, s);
@@ -390,7 +409,7 @@ archead_status archead_pack_create(const archead_desc *desc, void *stream, arche
   if (e == cudaSuccess && rr > 0) e = cudaMemcpyAsync(p->q_b, desc->corr_b, (size_t)d * rr, cudaMemcpyDefault, s);
   if (e == cudaSuccess && rr > 0) e = cudaMemcpyAsync(p->s_b, desc->corr_b_scale, G * rr * 2, cudaMemcpyDefault, s);
   if (e == cudaSuccess)
-    e = launch_build_layouts(p, t_codes, reinterpret_cast<uint16_t *>(t_scales), reinterpret_cast<int8_t *>(t_u),
+    e = launch_build_layouts(p, t_codes, t_scales, reinterpret_cast<uint16_t *>(t_srow), t_u,
                              reinterpret_cast<int8_t *>(t_a), reinterpret_cast<uint16_t *>(t_sa), s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   free_tmp();
@@ -485,8 +504,14 @@ archead_status archead_forward_host(archead_pack *pack, const void *x_host, int6
 int64_t archead_pack_bytes(const archead_pack *p) {
   if (!p) return -1;
   const int64_t V = p->V, d = p->d, rc = p->rc, rr = p->rr, G = p->G;
-  int64_t b = V * d / 2 + V * G * 2;          // INT4 residual + group scales
-  b += V * rc + rc * 2 + d * rc + rc * 2;     // core factors + column scales
+  int64_t b = V * d / 2;                      // INT4 residual
+  if (p->sc4) {
+    b += V * ((G + 1) / 2) + V * 2;           // 4-bit group-scale codes + row scales
+    b += V * ((5 * rc + 7) / 8);              // 5-bit core left codes
+  } else {
+    b += V * G * 2 + V * rc;                  // fp16 group scales + INT8 core left codes
+  }
+  b += rc * 2 + d * rc + rc * 2;              // core scales + right codes
   b += V * rr + (rr > 0 ? V * 2 : 0);         // correction left + row scales
   b += d * rr + G * rr * 2;                   // correction right + group scales
   return b;

@@ -1,649 +1,8 @@
-// Memory-bound decode kernel (M <= 16 tokens) of the packed LM-head forward
-// (paper, Section 3.2, Eq. 7; Appendix B: the core and correction paths are
-// evaluated separately and no dense head is formed).
-//
-// Persistent grid, one block per SM.  A unit of work is 512 vocabulary rows
-// (four 128-row tiles).  One producer warp streams each unit's INT4 codes,
-// group scales and low-rank codes with 1-D bulk TMA copies into a ring of
-// shared-memory stages (mbarrier full/empty pairs).  Eight consumer warps each
-// own four 16-row m-tiles.  The hidden states are staged once per block by
-// TMA and converted in place to fp16, each token scaled by a power of two that
-// keeps it in fp16 range (exact for bf16 inputs in the normal range).  Per
-// 16-wide k step a consumer turns one 32-bit word of offset-binary nibbles
-// into the four fp16 A-fragment registers of an m16n8k16 MMA (exact biased
-// integers, see unpack_int4x8_f16) and multiplies them with the hidden states
-// (B fragments, tokens on the 8-wide side), accumulating in fp32.  At the end
-// of every quantisation group the bias is removed and the partial sums are
-// promoted by that row's group scale in fp32.  The rank-r
-// branches follow as extra k steps: int8 codes of A_c (core) or A_w
-// (correction) times the bf16 hi/lo split of t = x V from the pre-pass, the
-// correction promoted by the row scale of A_w.  The pre-pass runs as the
-// preceding grid; this kernel starts streaming under programmatic dependent
-// launch and waits for the pre-pass only before the first rank-r stage.
-#include "device.cuh"
-#include "internal.h"
+// Host entry points of the decode kernel (decode_kernel.cuh); the INT8
+// format's instances compile here, the SC4 format's in decode_sc4.cu.
+#include "decode_kernel.cuh"
 
 namespace archead {
-
-constexpr int kDecWarps = 8;                      // consumer warps
-constexpr int kDecThreads = (kDecWarps + 1) * 32; // + producer warp
-constexpr int kDecTiles = 4;                      // 128-row tiles per unit
-constexpr int kDecMT = 4;                         // m-tiles per consumer warp (2 warps per tile)
-constexpr int kSmemLimit = 227 * 1024;
-
-// 64-wide chunks of d per ring stage, by number of 8-token n-tiles.  The
-// shared-memory plan and the kernel instance launched both take it from here.
-__host__ __device__ constexpr int stage_chunks(int NT) { return 2; }
-
-// Instances with two n-tiles (9..16 tokens) do not keep the hidden states in
-// shared memory (16 rows of d would take most of it, leaving too shallow a
-// ring to stream at full bandwidth).  Each residual stage instead carries the
-// matching 64-wide chunks of x for 16 tokens, loaded by a 2-D TMA copy, and
-// those instances multiply bf16 operands (no fp16 staging).  Their warps read
-// codes and x from the stage as they compute and release it afterwards (the
-// registers to copy a stage out first are not there with two n-tiles).
-__host__ __device__ constexpr bool streams_x(int NT) { return NT == 2; }
-constexpr int kXChunkBytes = 16 * kChunkK * 2;  // 16 tokens x 64 of d, bf16, 128-byte swizzle
-
-// Stage geometry for SC chunks (64 of d each) per stage.
-template <int SC, bool XS>
-struct StageGeom {
-  static constexpr int kCodeBytes = kDecTiles * SC * kChunkBytes;  // also holds 2*SC low-rank steps per tile
-  static constexpr int kScaleBytesPerTile = (SC * kChunkK / 32) * kTileRows * 2;  // up to SC*64/g groups (g >= 32)
-  static constexpr int kXOff = kCodeBytes + kDecTiles * kScaleBytesPerTile;       // a multiple of 1024
-  static constexpr int kBytes = kXOff + (XS ? SC * kXChunkBytes : 0);
-  static constexpr int kLrSteps = 2 * SC;  // 16-wide low-rank steps per stage (2 KB per tile each)
-};
-
-struct DecodePlan {
-  int stages, sc;
-  size_t xs_off, ts_off, xsum_off, bar_off, total;
-};
-
-__host__ __device__ __forceinline__ int xs_row_elems(int d_pad) { return d_pad + 8; }  // +16 B: rows on distinct banks
-
-// Shared memory: the stage ring, M rows of hidden states, the rank-r
-// fragments, the per-group sums of x, and the barriers.  The total leaves
-// room for one pre-pass block on the same SM (programmatic dependent launch
-// overlaps the two grids) whenever the stage ring still holds 96 KB.
-static DecodePlan decode_plan(int d_pad, int nls, int g, int M) {
-  DecodePlan pl{};
-  const int nt = M > 8 ? 2 : 1;
-  const bool xs = streams_x(nt);
-  pl.sc = stage_chunks(nt);
-  const size_t stage_bytes = pl.sc == 2 ? (xs ? StageGeom<2, true>::kBytes : StageGeom<2, false>::kBytes)
-                                        : (xs ? StageGeom<1, true>::kBytes : StageGeom<1, false>::kBytes);
-  const size_t xs_bytes = xs ? 0 : (size_t)M * xs_row_elems(d_pad) * 2;
-  const size_t ts_bytes = (size_t)nls * 1024;
-  const size_t xsum_bytes = ((size_t)2 * (d_pad / g) * kDecodeMaxTokens + kDecodeMaxTokens) * 4;
-  const size_t fixed = xs_bytes + ts_bytes + xsum_bytes + 256;
-  const size_t shared_cap = (size_t)kSmemLimit - prepass_smem(M) - 2048;
-  int st = 8;
-  while (st >= 2 && fixed + (size_t)st * stage_bytes > shared_cap) --st;
-  if (st < 2 || (size_t)st * stage_bytes < 96 * 1024) {  // too shallow a ring: give up co-residency
-    st = 8;
-    while (st >= 2 && fixed + (size_t)st * stage_bytes > (size_t)kSmemLimit) --st;
-  }
-  pl.stages = st;
-  pl.xs_off = (size_t)st * stage_bytes;
-  pl.ts_off = pl.xs_off + xs_bytes;
-  pl.xsum_off = pl.ts_off + ts_bytes;
-  pl.bar_off = pl.xsum_off + xsum_bytes;
-  pl.total = pl.bar_off + 256;
-  return pl;
-}
-
-// Residual group promotion with the operand bias removed:
-// acc += s_row * (part + nb_tok), nb = -(operand bias) * sum of x over the
-// group, separately for rows gq (bias 1032) and gq + 8 (bias 1152; s_hi
-// carries the 1/16 of those rows' operands).
-template <int NT>
-__device__ __forceinline__ void promote_res(float (&acc)[NT][4], const float (&part)[NT][4], float s_lo, float s_hi,
-                                            const float2 (&nb_lo)[NT], const float2 (&nb_hi)[NT]) {
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt) {
-    acc[nt][0] = fmaf(s_lo, part[nt][0] + nb_lo[nt].x, acc[nt][0]);
-    acc[nt][1] = fmaf(s_lo, part[nt][1] + nb_lo[nt].y, acc[nt][1]);
-    acc[nt][2] = fmaf(s_hi, part[nt][2] + nb_hi[nt].x, acc[nt][2]);
-    acc[nt][3] = fmaf(s_hi, part[nt][3] + nb_hi[nt].y, acc[nt][3]);
-  }
-}
-
-// acc += f_lo * part (rows gq) and f_hi * part (rows gq + 8).
-template <int NT>
-__device__ __forceinline__ void promote(float (&acc)[NT][4], const float (&part)[NT][4], float f_lo, float f_hi) {
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt) {
-    acc[nt][0] = fmaf(f_lo, part[nt][0], acc[nt][0]);
-    acc[nt][1] = fmaf(f_lo, part[nt][1], acc[nt][1]);
-    acc[nt][2] = fmaf(f_hi, part[nt][2], acc[nt][2]);
-    acc[nt][3] = fmaf(f_hi, part[nt][3], acc[nt][3]);
-  }
-}
-
-// NT: n-tiles of 8 tokens; SC: 64-wide chunks per stage; GS: 16-wide k steps per group.
-template <int NT, int SC, int GS>
-__global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_constant__ DecodeParams p, int stages,
-                                                                int xs_off, int ts_off, int xsum_off, int bar_off) {
-  constexpr bool kStreamX = streams_x(NT);
-  constexpr bool kF16 = !kStreamX;  // fp16 operands with x staged in shared memory
-  using Geom = StageGeom<SC, kStreamX>;
-  constexpr int SS = 4 * SC;  // 16-wide k steps per stage
-  // The kernel has no static shared memory, so the dynamic window starts on a
-  // 1 KB boundary, which the 128-byte-swizzled x boxes rely on (checked
-  // below).  Offsets from this base stay compile-time friendly; a rounded-up
-  // runtime base made the inner loops measurably slower.
-  extern __shared__ __align__(1024) uint8_t smem[];
-  if (kStreamX && (smem_u32(smem) & 1023u) != 0) {
-    if (threadIdx.x == 0) atomicOr(p.err, kErrLayout);
-    return;
-  }
-  uint16_t *xs_s = reinterpret_cast<uint16_t *>(smem + xs_off);
-  const uint32_t *ts_s = reinterpret_cast<const uint32_t *>(smem + ts_off);
-  // [group][16 tokens] -1032 * sum of x, then the same with -1152, then the
-  // 16 tokens' scale factors (powers of two) that undo the fp16 staging scale.
-  float *xsum_s = reinterpret_cast<float *>(smem + xsum_off);
-  uint64_t *full = reinterpret_cast<uint64_t *>(smem + bar_off);
-  uint64_t *empty = full + 8;
-  uint64_t *xbar = full + 16;
-  uint64_t *tbar = full + 17;
-  volatile int *abort_flag = reinterpret_cast<volatile int *>(full + 18);
-
-  const int warp = threadIdx.x >> 5;
-  const int lane = threadIdx.x & 31;
-  const int KC = p.d_pad / kChunkK;
-  const int res_stages = KC / SC;
-  const int lr_stages = (p.nls + Geom::kLrSteps - 1) / Geom::kLrSteps;
-  const int num_units = (p.num_tiles + kDecTiles - 1) / kDecTiles;
-  const int xrow = xs_row_elems(p.d_pad);
-
-  // Columns [d, d_pad) of the hidden states meet zero codes; zero them so
-  // that no stale pattern (a NaN) reaches the accumulators.
-  if (!kStreamX && p.d < p.d_pad) {
-    const int per_row = (p.d_pad - p.d) / 8;  // uint4 per row
-    for (int e = threadIdx.x; e < p.M * per_row; e += blockDim.x) {
-      uint4 *dst = reinterpret_cast<uint4 *>(smem + xs_off + (size_t)(e / per_row) * xrow * 2 + (size_t)p.d * 2);
-      dst[e % per_row] = make_uint4(0, 0, 0, 0);
-    }
-  }
-  if (threadIdx.x == 0) {
-    for (int i = 0; i < stages; ++i) {
-      mbar_init(&full[i], 1);
-      mbar_init(&empty[i], kDecWarps);
-    }
-    mbar_init(xbar, 1);
-    mbar_init(tbar, 1);
-    *abort_flag = 0;
-    fence_mbar_init();
-  }
-  __syncthreads();
-
-  if (warp == kDecWarps) {
-    // ---------------- producer warp ----------------
-    // The whole warp runs the loop (voted waits keep it warp-uniform) and one
-    // elected lane issues the copies: a single-lane loop issues bulk copies
-    // several times more slowly.
-    const bool leader = elect_one();
-    // The head is read once per forward: keep it from evicting the small
-    // data the pre-pass grid reads at the same time.
-    const uint64_t stream_policy = make_evict_first_policy();
-    if (!kStreamX && leader) {
-      mbar_arrive_expect_tx(xbar, (uint32_t)(p.M * p.d * 2));
-      for (int m = 0; m < p.M; ++m)
-        bulk_g2s(smem + xs_off + (size_t)m * xrow * 2, p.x + (size_t)(p.m0 + m) * p.d, (uint32_t)(p.d * 2), xbar);
-    }
-    bool t_loaded = false;
-    int it = 0;
-    for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x) {
-      const int ntile = min(kDecTiles, p.num_tiles - kDecTiles * unit);
-      for (int s = 0; s < res_stages + lr_stages; ++s, ++it) {
-        const int st = it % stages;
-        if (s == res_stages && !t_loaded) {
-          // The rank-r fragments come from the pre-pass grid.
-          asm volatile("griddepcontrol.wait;\n" ::: "memory");
-          if (leader) {
-            mbar_arrive_expect_tx(tbar, (uint32_t)(p.nls * 1024));
-            bulk_g2s(smem + ts_off, p.ts, (uint32_t)(p.nls * 1024), tbar);
-          }
-          t_loaded = true;
-        }
-        if (!mbar_wait_warp(&empty[st], ((it / stages) & 1) ^ 1, p.wait_budget, abort_flag, p.err))
-          goto producer_abort;
-        uint8_t *buf = smem + (size_t)st * Geom::kBytes;
-        if (!leader) {
-        } else if (s < res_stages) {
-          const int kc0 = s * SC;
-          const int g0 = (kc0 * kChunkK) / p.g;
-          const int g1 = ((kc0 + SC) * kChunkK - 1) / p.g;
-          const int ng = g1 - g0 + 1;
-          mbar_arrive_expect_tx(&full[st],
-                                (uint32_t)(ntile * (SC * kChunkBytes + ng * kTileRows * 2) + (kStreamX ? SC * kXChunkBytes : 0)));
-          if (kStreamX) {
-            for (int c = 0; c < SC; ++c)
-              tma_load_2d(buf + Geom::kXOff + c * kXChunkBytes, &p.tmap_x, (kc0 + c) * kChunkK, p.m0, &full[st]);
-          }
-          for (int t = 0; t < ntile; ++t) {
-            const int64_t vt = (int64_t)kDecTiles * unit + t;
-            bulk_g2s_hint(buf + t * SC * kChunkBytes, p.codes + (vt * KC + kc0) * kChunkBytes, SC * kChunkBytes,
-                          &full[st], stream_policy);
-            bulk_g2s_hint(buf + Geom::kCodeBytes + t * Geom::kScaleBytesPerTile, p.scales + (vt * p.G_pad + g0) * kTileRows,
-                          ng * kTileRows * 2, &full[st], stream_policy);
-          }
-        } else {
-          const int ls0 = (s - res_stages) * Geom::kLrSteps;
-          const int nl = min(Geom::kLrSteps, p.nls - ls0);
-          const bool last = (s == res_stages + lr_stages - 1);
-          mbar_arrive_expect_tx(&full[st], (uint32_t)(ntile * (nl * kLrStepBytes + (last ? kTileRows * 2 : 0))));
-          for (int t = 0; t < ntile; ++t) {
-            const int64_t vt = (int64_t)kDecTiles * unit + t;
-            bulk_g2s_hint(buf + t * Geom::kLrSteps * kLrStepBytes, p.lr_codes + (vt * p.nls + ls0) * kLrStepBytes,
-                          nl * kLrStepBytes, &full[st], stream_policy);
-            if (last)
-              bulk_g2s(buf + Geom::kCodeBytes + t * Geom::kScaleBytesPerTile, p.s_a + vt * kTileRows, kTileRows * 2,
-                       &full[st]);
-          }
-        }
-        __syncwarp();
-      }
-    }
-    return;
-  producer_abort:
-    // Let copies already issued land before the block exits.
-    for (int k = 1; k <= stages && it - k >= 0; ++k) {
-      const int j = it - k;
-      mbar_wait_warp(&full[j % stages], (j / stages) & 1, p.wait_budget, nullptr, p.err);
-    }
-    if (!kStreamX) mbar_wait_warp(xbar, 0, p.wait_budget, nullptr, p.err);
-    if (t_loaded) mbar_wait_warp(tbar, 0, p.wait_budget, nullptr, p.err);
-    return;
-  }
-
-  // ---------------- consumer warps ----------------
-  const int tsel = warp / (8 / kDecMT);              // tile of the unit
-  const int mi0 = (warp % (8 / kDecMT)) * kDecMT;    // first of the warp's m-tiles in that tile
-  const int gq = lane >> 2, cq = lane & 3;
-  const int ng = p.d_pad / p.g;
-  float *tscale = xsum_s + 2 * ng * kDecodeMaxTokens;
-  if (kStreamX) {
-    // Per-group sums of x for removing the bf16 operand bias (136), read
-    // straight from global memory; no staging scale.
-    for (int e = threadIdx.x; e < ng * kDecodeMaxTokens; e += kDecWarps * 32) {
-      const int grp = e / kDecodeMaxTokens, m = e % kDecodeMaxTokens;
-      float sum = 0.f;
-      if (m < p.M && grp * p.g < p.d) {
-        const uint4 *src = reinterpret_cast<const uint4 *>(p.x + (int64_t)(p.m0 + m) * p.d + (int64_t)grp * p.g);
-        for (int q = 0; q < p.g / 8; ++q) {
-          const uint4 v = src[q];
-          sum += bf16_lo(v.x) + bf16_hi(v.x) + bf16_lo(v.y) + bf16_hi(v.y);
-          sum += bf16_lo(v.z) + bf16_hi(v.z) + bf16_lo(v.w) + bf16_hi(v.w);
-        }
-      }
-      xsum_s[e] = -kInt4Bias * sum;
-      xsum_s[ng * kDecodeMaxTokens + e] = -kInt4Bias * sum;
-    }
-    if (threadIdx.x < kDecodeMaxTokens) tscale[threadIdx.x] = 1.f;
-    asm volatile("bar.sync 1, %0;\n" ::"r"(kDecWarps * 32) : "memory");  // consumer warps only
-  } else {
-    const bool ok = mbar_wait_warp(xbar, 0, p.wait_budget, abort_flag, p.err);
-    if (ok) {
-      // Per-token power of two 2^-e that brings max |x| into [2^14, 2^15)
-      // (fp16 range, and small tokens away from fp16 subnormals); tscale[m]
-      // = 2^e undoes it after the residual.
-      for (int m = warp; m < kDecodeMaxTokens; m += kDecWarps) {
-        uint32_t mx = 0;
-        if (m < p.M) {
-          const uint32_t *row = reinterpret_cast<const uint32_t *>(xs_s + m * xrow);
-          for (int k = lane; k < p.d_pad / 2; k += 32) {
-            const uint32_t v = row[k];
-            mx = max(mx, max(v & 0x7FFFu, (v >> 16) & 0x7FFFu));
-          }
-        }
-        mx = __reduce_max_sync(0xffffffffu, mx);
-        const int ex = (int)(mx >> 7);             // biased bf16 exponent of the largest |x|
-        const int e = max(ex - 141, -126);       // max |x| < 2^(ex-126); 2^-e of it lies below 2^15
-        if (lane == 0) tscale[m] = __uint_as_float((uint32_t)(127 + e) << 23);
-      }
-      asm volatile("bar.sync 1, %0;\n" ::"r"(kDecWarps * 32) : "memory");
-      // Convert each token's row to fp16 in place, group by group, and sum
-      // the values the MMAs will see (for removing the operand bias).
-      for (int e = threadIdx.x; e < ng * kDecodeMaxTokens; e += kDecWarps * 32) {
-        const int grp = e / kDecodeMaxTokens, m = e % kDecodeMaxTokens;
-        float sum = 0.f;
-        if (m < p.M) {
-          const float inv = 1.f / tscale[m];  // exact: a power of two
-          uint32_t *row = reinterpret_cast<uint32_t *>(xs_s + m * xrow + grp * p.g);
-          for (int k = 0; k < p.g / 2; ++k) {
-            const uint32_t v = row[k];
-            const __half2 h = __floats2half2_rn(bf16_lo(v) * inv, bf16_hi(v) * inv);
-            row[k] = *reinterpret_cast<const uint32_t *>(&h);
-            sum += __low2float(h);
-            sum += __high2float(h);
-          }
-        }
-        xsum_s[e] = -kF16BiasLo * sum;
-        xsum_s[ng * kDecodeMaxTokens + e] = -kF16BiasHi * sum;
-      }
-    }
-    asm volatile("bar.sync 1, %0;\n" ::"r"(kDecWarps * 32) : "memory");  // consumer warps only
-    if (!ok) return;
-  }
-  // Factors that undo the staging scale for this lane's two token columns.
-  float2 unscale[NT];
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt) unscale[nt] = make_float2(tscale[8 * nt + 2 * cq], tscale[8 * nt + 2 * cq + 1]);
-  // B-fragment bases: token 8*nt + gq (clamped to the M rows held; the extra
-  // columns are never stored), column 2*cq (+ 16 per k step, + 8 for b1).
-  const uint16_t *xb[NT];
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt) xb[nt] = kStreamX ? nullptr : xs_s + min(8 * nt + gq, p.M - 1) * xrow + 2 * cq;
-  bool t_ready = false;
-
-  int st = 0;     // ring slot
-  uint32_t ph = 0;  // its phase parity
-  for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x) {
-    const int ntile = min(kDecTiles, p.num_tiles - kDecTiles * unit);
-    const bool active = tsel < ntile;
-    float acc[kDecMT][NT][4];
-    float part[kDecMT][NT][4];  // one group's sums; each group's first MMA starts from zero
-#pragma unroll
-    for (int a = 0; a < kDecMT; ++a)
-#pragma unroll
-      for (int b = 0; b < NT; ++b)
-#pragma unroll
-        for (int c = 0; c < 4; ++c) acc[a][b][c] = part[a][b][c] = 0.f;
-
-    // Residual: INT4 codes, promoted per group.  With x resident, each warp
-    // copies its share of a stage (codes and group scales) to registers and
-    // releases the slot at once, so the producer can refill it while the warp
-    // computes; with x streamed, it releases the slot after its k steps.
-    constexpr int NGS = GS <= SS ? SS / GS : 1;  // groups whose scales a stage carries
-    for (int s = 0; s < res_stages; ++s) {
-      if (!mbar_wait_warp(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
-      uint4 w[kStreamX ? 1 : SC][kDecMT];
-      float s_lo[NGS][kDecMT], s_hi[NGS][kDecMT];
-      const uint8_t *sbuf = smem + (size_t)st * Geom::kBytes;
-      const uint8_t *cb = sbuf + tsel * SC * kChunkBytes + mi0 * 512 + lane * 16;
-      if (active) {
-        const uint16_t *sc = reinterpret_cast<const uint16_t *>(sbuf + Geom::kCodeBytes + tsel * Geom::kScaleBytesPerTile) +
-                             mi0 * 16 + gq;
-        if (!kStreamX) {
-#pragma unroll
-          for (int c = 0; c < (kStreamX ? 1 : SC); ++c)
-#pragma unroll
-            for (int mt = 0; mt < kDecMT; ++mt)
-              w[c][mt] = *reinterpret_cast<const uint4 *>(cb + c * kChunkBytes + mt * 512);
-        }
-#pragma unroll
-        for (int gi = 0; gi < NGS; ++gi)
-#pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt) {
-            s_lo[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16]);
-            s_hi[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16 + 8]) * (kF16 ? 0.0625f : 1.f);  // fp16: x16
-          }
-      }
-      const int st_done = st;
-      if (!kStreamX || !active) {
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&empty[st]);
-      }
-      if (++st == stages) st = 0, ph ^= 1;
-      if (!active) continue;
-      const int kbase = s * SS * 16;
-#pragma unroll
-      for (int c = 0; c < SC; ++c) {
-        if (kStreamX) {
-#pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt)
-            w[0][mt] = *reinterpret_cast<const uint4 *>(cb + c * kChunkBytes + mt * 512);
-        }
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int ks = c * 4 + j;  // k step within the stage
-          uint32_t b[NT][2];
-#pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
-            if (kStreamX) {
-              // Token 8*nt + gq, k = 16*ks + 2*cq (+8): 128-byte rows, 16-byte
-              // chunk index XOR (row % 8) = gq.
-              const uint8_t *xr = sbuf + Geom::kXOff + c * kXChunkBytes + (8 * nt + gq) * 128 + 4 * cq;
-              b[nt][0] = *reinterpret_cast<const uint32_t *>(xr + (((2 * j) ^ gq) << 4));
-              b[nt][1] = *reinterpret_cast<const uint32_t *>(xr + (((2 * j + 1) ^ gq) << 4));
-            } else {
-              const uint16_t *q = xb[nt] + kbase + ks * 16;
-              b[nt][0] = *reinterpret_cast<const uint32_t *>(q);
-              b[nt][1] = *reinterpret_cast<const uint32_t *>(q + 8);
-            }
-          }
-#pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt) {
-            const uint4 wv = w[kStreamX ? 0 : c][mt];
-            const uint32_t word = j == 0 ? wv.x : j == 1 ? wv.y : j == 2 ? wv.z : wv.w;
-            uint32_t a[4];
-            if (kF16)
-              unpack_int4x8_f16(word, a);
-            else
-              unpack_int4x8_biased(word, a);
-            // First k step of a group: compile-time when groups fit in a stage.
-            const bool first = GS <= SS ? (ks % GS == 0) : (ks == 0 && (s % (GS / SS)) == 0);
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-              if (kF16) {
-                if (first)
-                  mma_f16_16816_zero(part[mt][nt], a, b[nt][0], b[nt][1]);
-                else
-                  mma_f16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
-              } else {
-                if (first)
-                  mma_bf16_16816_zero(part[mt][nt], a, b[nt][0], b[nt][1]);
-                else
-                  mma_bf16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
-              }
-            }
-          }
-          // Group boundary: compile-time inside a stage when GS <= SS; every
-          // GS/SS stages otherwise.
-          const bool boundary = GS <= SS ? ((ks + 1) % GS == 0) : (ks == SS - 1 && ((s + 1) % (GS / SS)) == 0);
-          if (boundary) {
-            const int gi = GS <= SS ? ks / GS : 0;                               // group within the stage
-            const int ggl = GS <= SS ? s * (SS / GS) + ks / GS : s / (GS / SS);  // group index along d
-            float2 nb_lo[NT], nb_hi[NT];
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-              const int o = ggl * kDecodeMaxTokens + 8 * nt + 2 * cq;
-              nb_lo[nt] = *reinterpret_cast<const float2 *>(xsum_s + o);
-              nb_hi[nt] = *reinterpret_cast<const float2 *>(xsum_s + ng * kDecodeMaxTokens + o);
-            }
-#pragma unroll
-            for (int mt = 0; mt < kDecMT; ++mt)
-              promote_res<NT>(acc[mt], part[mt], s_lo[gi][mt], s_hi[gi][mt], nb_lo, nb_hi);
-          }
-        }
-      }
-      if (kStreamX) {
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&empty[st_done]);
-      }
-    }
-
-    // Back to the hidden states' own scale (exact: powers of two).
-#pragma unroll
-    for (int a = 0; a < (kF16 ? kDecMT : 0); ++a)
-#pragma unroll
-      for (int b = 0; b < NT; ++b) {
-        acc[a][b][0] *= unscale[b].x;
-        acc[a][b][1] *= unscale[b].y;
-        acc[a][b][2] *= unscale[b].x;
-        acc[a][b][3] *= unscale[b].y;
-      }
-
-    // Rank-r branches as extra k steps (core: factor 1; correction: row scale
-    // of A_w), with the same copy-then-release of each stage.
-#pragma unroll
-    for (int a = 0; a < kDecMT; ++a)
-#pragma unroll
-      for (int b = 0; b < NT; ++b)
-#pragma unroll
-        for (int c = 0; c < 4; ++c) part[a][b][c] = 0.f;
-    for (int s = 0; s < lr_stages; ++s) {
-      if (!t_ready) {
-        if (!mbar_wait_warp(tbar, 0, p.wait_budget, abort_flag, p.err)) return;
-        t_ready = true;
-      }
-      if (!mbar_wait_warp(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
-      const int ls0 = s * Geom::kLrSteps;
-      const int nl = min(Geom::kLrSteps, p.nls - ls0);
-      const bool last_stage = s == lr_stages - 1;
-      uint2 lw[Geom::kLrSteps][kDecMT];
-      float a_lo[kDecMT], a_hi[kDecMT];
-      if (active) {
-        const uint8_t *buf = smem + (size_t)st * Geom::kBytes;
-#pragma unroll
-        for (int l = 0; l < Geom::kLrSteps; ++l)
-#pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt)
-            if (l < nl)
-              lw[l][mt] = *reinterpret_cast<const uint2 *>(
-                  buf + ((size_t)(tsel * Geom::kLrSteps + l) * 8 + mi0 + mt) * 256 + lane * 8);
-        const uint16_t *sa = reinterpret_cast<const uint16_t *>(buf + Geom::kCodeBytes + tsel * Geom::kScaleBytesPerTile);
-#pragma unroll
-        for (int mt = 0; mt < kDecMT; ++mt) {
-          const int r = (mi0 + mt) * 16 + gq;
-          a_lo[mt] = last_stage ? fp16_bits_to_f32(sa[r]) : 0.f;
-          a_hi[mt] = last_stage ? fp16_bits_to_f32(sa[r + 8]) : 0.f;
-        }
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&empty[st]);
-      if (++st == stages) st = 0, ph ^= 1;
-      if (!active) continue;
-#pragma unroll
-      for (int l = 0; l < Geom::kLrSteps; ++l) {
-        if (l >= nl) break;
-        const int ls = ls0 + l;
-        uint32_t bh[NT][2], bl[NT][2];
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-          const uint2 h2 = *reinterpret_cast<const uint2 *>(ts_s + ((((size_t)ls * 2 + 0) * 2 + nt) * 32 + lane) * 2);
-          const uint2 l2 = *reinterpret_cast<const uint2 *>(ts_s + ((((size_t)ls * 2 + 1) * 2 + nt) * 32 + lane) * 2);
-          bh[nt][0] = h2.x;
-          bh[nt][1] = h2.y;
-          bl[nt][0] = l2.x;
-          bl[nt][1] = l2.y;
-        }
-#pragma unroll
-        for (int mt = 0; mt < kDecMT; ++mt) {
-          uint32_t a[4];
-          unpack_int8x8(lw[l][mt].x, lw[l][mt].y, a);
-#pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
-            mma_bf16_16816(part[mt][nt], a, bh[nt][0], bh[nt][1]);
-            mma_bf16_16816(part[mt][nt], a, bl[nt][0], bl[nt][1]);
-          }
-        }
-        if (ls + 1 == p.nls_core || ls + 1 == p.nls) {
-          const bool corr = ls + 1 == p.nls && p.nls > p.nls_core;  // the correction ends with the last stage
-#pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt) {
-            promote<NT>(acc[mt], part[mt], corr ? a_lo[mt] : 1.f, corr ? a_hi[mt] : 1.f);
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-              for (int c = 0; c < 4; ++c) part[mt][nt][c] = 0.f;
-          }
-        }
-      }
-    }
-
-    // Epilogue.  acc[mt][nt][i]: row 16*(mi0+mt) + gq + 8*(i/2), token 8*nt + 2*cq + i%2.
-    const int64_t row_base = ((int64_t)kDecTiles * unit + tsel) * kTileRows;
-    if (p.out) {
-      if (active) {
-#pragma unroll
-        for (int mt = 0; mt < kDecMT; ++mt)
-#pragma unroll
-          for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const int64_t row = row_base + (mi0 + mt) * 16 + gq + 8 * (i >> 1);
-              const int tok = nt * 8 + 2 * cq + (i & 1);
-              if (row < p.V && tok < p.M) {
-                const int64_t o = (int64_t)(p.m0 + tok) * p.V + row;
-                if (p.out_fp32)
-                  reinterpret_cast<float *>(p.out)[o] = acc[mt][nt][i];
-                else
-                  reinterpret_cast<__nv_bfloat16 *>(p.out)[o] = __float2bfloat16_rn(acc[mt][nt][i]);
-              }
-            }
-      }
-    } else if (p.argmax) {
-      // Greedy partials: per (unit, warp, token) the largest logit and its
-      // row (the lowest row on ties), as (value, row bits).
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int tl = 0; tl < 2; ++tl) {
-          const int tok = nt * 8 + 2 * cq + tl;
-          float bv = -INFINITY;
-          int bi = 0x7fffffff;
-#pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt)
-#pragma unroll
-            for (int ih = 0; ih < 2; ++ih) {
-              const int64_t row = row_base + (mi0 + mt) * 16 + gq + 8 * ih;
-              const float v = acc[mt][nt][ih * 2 + tl];
-              if (active && row < p.V && (v > bv || (v == bv && (int)row < bi))) {
-                bv = v;
-                bi = (int)row;
-              }
-            }
-#pragma unroll
-          for (int off = 4; off < 32; off <<= 1) {
-            const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
-            const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-            if (ov > bv || (ov == bv && oi < bi)) {
-              bv = ov;
-              bi = oi;
-            }
-          }
-          if (gq == 0 && tok < p.M)
-            p.ce_part[((int64_t)unit * kDecWarps + warp) * p.M_total + p.m0 + tok] = make_float2(bv, __int_as_float(bi));
-        }
-    } else {
-      // Cross-entropy partials: per (unit, warp, token) running max and sum of exp.
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int tl = 0; tl < 2; ++tl) {
-          const int tok = nt * 8 + 2 * cq + tl;
-          const int tgt = tok < p.M ? p.targets[p.m0 + tok] : -1;
-          float vals[2 * kDecMT];
-          float mx = -INFINITY;
-#pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt)
-#pragma unroll
-            for (int ih = 0; ih < 2; ++ih) {
-              const int64_t row = row_base + (mi0 + mt) * 16 + gq + 8 * ih;
-              const bool ok = active && row < p.V;
-              const float v = ok ? acc[mt][nt][ih * 2 + tl] : -INFINITY;
-              vals[mt * 2 + ih] = v;
-              mx = fmaxf(mx, v);
-              if (ok && row == tgt) p.ce_tlogit[p.m0 + tok] = v;
-            }
-          float sum = 0.f;
-#pragma unroll
-          for (int q = 0; q < 2 * kDecMT; ++q) sum += (vals[q] == -INFINITY) ? 0.f : __expf(vals[q] - mx);
-          LsePair lp{mx, sum};
-#pragma unroll
-          for (int off = 4; off < 32; off <<= 1) {
-            LsePair o{__shfl_xor_sync(0xffffffffu, lp.m, off), __shfl_xor_sync(0xffffffffu, lp.s, off)};
-            lp = lse_merge(lp, o);
-          }
-          if (gq == 0 && tok < p.M)
-            p.ce_part[((int64_t)unit * kDecWarps + warp) * p.M_total + p.m0 + tok] = make_float2(lp.m, lp.s);
-        }
-    }
-  }
-}
 
 int decode_num_units(const archead_pack *p) { return (p->num_tiles + kDecTiles - 1) / kDecTiles; }
 
@@ -651,50 +10,11 @@ int decode_parts_per_unit() { return kDecWarps; }
 
 bool decode_supported(int d_pad, int nls, int g) { return decode_plan(d_pad, nls, g, kDecodeMaxTokens).stages >= 2; }
 
-template <int NT, int SC, int GS>
-static cudaError_t launch_t(const DecodeParams &dp, int grid, cudaStream_t s, const DecodePlan &pl, bool pdl) {
-  auto kern = decode_kernel<NT, SC, GS>;
-  static int smem_set = 0;  // largest dynamic shared memory opted in so far for this instance
-  if ((int)pl.total > smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.total);
-    if (e != cudaSuccess) return e;
-    smem_set = (int)pl.total;
-  }
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(kDecThreads);
-  cfg.dynamicSmemBytes = pl.total;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, kern, dp, pl.stages, (int)pl.xs_off, (int)pl.ts_off, (int)pl.xsum_off,
-                            (int)pl.bar_off);
-}
-
-template <int NT, int SC>
-static cudaError_t launch_g(const DecodeParams &dp, int grid, cudaStream_t s, const DecodePlan &pl, bool pdl) {
-  switch (dp.g) {
-    case 32: return launch_t<NT, SC, 2>(dp, grid, s, pl, pdl);
-    case 64: return launch_t<NT, SC, 4>(dp, grid, s, pl, pdl);
-    case 128: return launch_t<NT, SC, 8>(dp, grid, s, pl, pdl);
-    case 256: return launch_t<NT, SC, 16>(dp, grid, s, pl, pdl);
-  }
-  return cudaErrorInvalidValue;
-}
+extern template cudaError_t launch_decode_fmt<true>(const DecodeParams &, int, cudaStream_t, bool);
+template cudaError_t launch_decode_fmt<false>(const DecodeParams &, int, cudaStream_t, bool);
 
 cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool pdl) {
-  const DecodePlan pl = decode_plan(dp.d_pad, dp.nls, dp.g, dp.M);
-  if (pl.stages < 2) return cudaErrorInvalidValue;
-  static_assert(stage_chunks(1) >= 1 && stage_chunks(2) >= 1, "stage width");
-  if ((dp.NT == 1) != (dp.M <= 8) || pl.sc != stage_chunks(dp.NT)) return cudaErrorInvalidValue;
-  if (dp.NT == 1) return launch_g<1, stage_chunks(1)>(dp, grid, s, pl, pdl);
-  static_assert(streams_x(2) && !streams_x(1), "two n-tiles stream x");
-  DecodeParams dx = dp;
-  if (!make_tma_map_bf16(&dx.tmap_x, dp.x, dp.M_total, dp.d, 16)) return cudaErrorInvalidValue;
-  return launch_g<2, stage_chunks(2)>(dx, grid, s, pl, pdl);
+  return dp.sc4 ? launch_decode_fmt<true>(dp, grid, s, pdl) : launch_decode_fmt<false>(dp, grid, s, pdl);
 }
 
 }  // namespace archead

@@ -15,6 +15,13 @@
 //  Residual scales: [vt][G_PAD][128] fp16 bits (row within tile fastest),
 //  G_PAD = D_PAD/g; scales of padding groups and rows are zero.
 //
+//  The paper's packed format (ARCHEAD_FORMAT_SC4) replaces them by 4-bit
+//  group-scale codes and one fp16 scale per row: codes [vt][G_PAD2][128]
+//  bytes, G_PAD2 = ceil(G_PAD/2), byte j of a row holding groups 2j (low
+//  nibble) and 2j+1; row scales [V_pad] fp16 (zero on padding rows).  The
+//  group scale is s_row * (q + 1).  Its 5-bit core left codes are widened
+//  into the low-rank codes below at pack time.
+//
 //  Low-rank codes: the extended rank axis kk in [0, LR) with LR = RCP + RRP,
 //  RCP = r_c rounded up to 32, RRP = r_r rounded up to 32: kk < RCP is
 //  core_u[:, kk], kk >= RCP is corr_a[:, kk - RCP] (zero beyond the rank).
@@ -48,13 +55,16 @@ constexpr int64_t kDefaultWaitBudget = 2000000000LL;  // cycles, about one secon
 struct DecodeParams {
   CUtensorMap tmap_x;   // x [M_total][d] bf16, box 64 x 16 rows (kernel instances that stream x; M > 8)
   const uint8_t *codes;
-  const uint16_t *scales;
+  const uint16_t *scales;   // fp16 group scales (INT8 format)
+  const uint8_t *scodes;    // 4-bit group-scale codes (SC4 format)
+  const uint16_t *s_row;    // residual row scales (SC4 format)
   const uint8_t *lr_codes;
   const uint16_t *s_a;
   const uint16_t *x;    // hidden states [M_total][d] bf16 (this chunk starts at row m0)
   const uint32_t *ts;   // t hi/lo fragments for this token chunk
   int64_t V;
   int num_tiles, d, d_pad, G_pad, g, nls, nls_core;
+  int sc4, G_pad2;      // SC4 format flag; byte rows of scale codes per tile
   int M;                // tokens in this chunk (1..16)
   int m0;               // index of the chunk's first token
   int NT;               // n-tiles of 8 tokens (1 or 2)
@@ -99,9 +109,13 @@ struct archead_pack {
   int d = 0, rc = 0, rr = 0, g = 0, G = 0, rcp = 0, rrp = 0, lr = 0, nls = 0, nls_core = 0;
   int d_pad = 0, G_pad = 0;  // d rounded up to 128, and its group count
   int num_tiles = 0;
+  int sc4 = 0;               // ARCHEAD_FORMAT_SC4
+  int G_pad2 = 0;            // ceil(G_pad / 2): bytes of scale codes per row (SC4)
   // device buffers owned by the pack
   uint8_t *codes = nullptr;
-  uint16_t *scales = nullptr;
+  uint16_t *scales = nullptr;  // INT8 format
+  uint8_t *scodes = nullptr;   // SC4 format
+  uint16_t *s_row = nullptr;   // SC4 format
   uint8_t *lr_codes = nullptr;
   uint16_t *s_a = nullptr;
   int8_t *q_v = nullptr, *q_b = nullptr;
@@ -125,9 +139,11 @@ struct archead_pack {
 namespace archead {
 
 // Kernel launchers (each returns the launch's cudaError_t).
-cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, const uint16_t *res_scales,
-                                 const int8_t *core_u, const int8_t *corr_a, const uint16_t *corr_a_scale,
-                                 cudaStream_t s);
+// res_scales and core_u are the canonical arrays of the pack's format (SC4:
+// 4-bit scale codes and 5-bit core codes; row_scale its residual row scales).
+cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, const void *res_scales,
+                                 const uint16_t *row_scale, const void *core_u, const int8_t *corr_a,
+                                 const uint16_t *corr_a_scale, cudaStream_t s);
 cudaError_t launch_debug_dequant(const archead_pack *p, int comp, int64_t row0, int64_t nrows, float *out,
                                  cudaStream_t s);
 cudaError_t launch_prepass(const PrepassParams &pp, cudaStream_t s, archead_pack *p);

@@ -50,9 +50,35 @@ __global__ void build_res_scales_kernel(const uint16_t *__restrict__ src, uint16
   }
 }
 
-// One block per (tile, 16-wide step of the extended rank axis).
-__global__ void build_lr_codes_kernel(const int8_t *__restrict__ core_u, const int8_t *__restrict__ corr_a,
-                                      uint8_t *__restrict__ dst, int64_t V, int rc, int rr, int rcp, int nls) {
+// SC4 group-scale codes: canonical [V][ceil(G/2)] bytes -> [vt][G_pad2][128].
+// Nibbles of groups past G (padding groups) are cleared.
+__global__ void build_scale_codes_kernel(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst, int64_t V,
+                                         int64_t V_pad, int G, int G_pad2) {
+  const int nbc = (G + 1) / 2;
+  const int64_t total = V_pad * G_pad2;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = i % kTileRows;
+    const int j = (int)((i / kTileRows) % G_pad2);
+    const int64_t row = (i / ((int64_t)kTileRows * G_pad2)) * kTileRows + r;
+    uint8_t b = (row < V && j < nbc) ? src[row * nbc + j] : (uint8_t)0;
+    if (2 * j + 1 >= G) b &= 0x0F;
+    dst[i] = b;
+  }
+}
+
+// Signed 5-bit code j of a row of ceil(5 r_c / 8) bytes (bits 5j..5j+4, LSB first).
+__device__ __forceinline__ int int5_code(const uint8_t *row, int j) {
+  const int bit = 5 * j, b = bit >> 3, sh = bit & 7;
+  uint32_t v = (uint32_t)row[b] >> sh;
+  if (sh > 3) v |= (uint32_t)row[b + 1] << (8 - sh);
+  v &= 31u;
+  return v >= 16 ? (int)v - 32 : (int)v;
+}
+
+// One block per (tile, 16-wide step of the extended rank axis).  core_u is
+// int8 [V][r_c], or with u5 != 0 the SC4 5-bit codes [V][ceil(5 r_c / 8)].
+__global__ void build_lr_codes_kernel(const void *__restrict__ core_u, const int8_t *__restrict__ corr_a,
+                                      uint8_t *__restrict__ dst, int64_t V, int rc, int rr, int rcp, int nls, int u5) {
   const int vt = blockIdx.x / nls;
   const int ls = blockIdx.x % nls;
   uint8_t *out = dst + ((int64_t)vt * nls + ls) * kLrStepBytes;
@@ -65,7 +91,9 @@ __global__ void build_lr_codes_kernel(const int8_t *__restrict__ core_u, const i
     int code = 0;
     if (row < V) {
       if (kk < rcp) {
-        if (kk < rc) code = core_u[row * rc + kk];
+        if (kk < rc)
+          code = u5 ? int5_code(static_cast<const uint8_t *>(core_u) + row * ((5 * rc + 7) / 8), kk)
+                    : static_cast<const int8_t *>(core_u)[row * rc + kk];
       } else if (kk - rcp < rr) {
         code = corr_a[row * rr + (kk - rcp)];
       }
@@ -99,15 +127,22 @@ __global__ void build_lr_t_kernel(const int8_t *__restrict__ q_v, const int8_t *
   }
 }
 
-cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, const uint16_t *res_scales,
-                                 const int8_t *core_u, const int8_t *corr_a, const uint16_t *corr_a_scale,
-                                 cudaStream_t s) {
+cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, const void *res_scales,
+                                 const uint16_t *row_scale, const void *core_u, const int8_t *corr_a,
+                                 const uint16_t *corr_a_scale, cudaStream_t s) {
   const int KC = p->d_pad / kChunkK;
   build_res_codes_kernel<<<p->num_tiles * KC, 256, 0, s>>>(res_codes, p->codes, p->V, p->d, p->d_pad);
-  build_res_scales_kernel<<<1024, 256, 0, s>>>(res_scales, p->scales, p->V, p->V_pad, p->G, p->G_pad);
+  if (p->sc4) {
+    build_scale_codes_kernel<<<1024, 256, 0, s>>>(static_cast<const uint8_t *>(res_scales), p->scodes, p->V, p->V_pad,
+                                                  p->G, p->G_pad2);
+    build_row_scales_kernel<<<256, 256, 0, s>>>(row_scale, p->s_row, p->V, p->V_pad);
+  } else {
+    build_res_scales_kernel<<<1024, 256, 0, s>>>(static_cast<const uint16_t *>(res_scales), p->scales, p->V, p->V_pad,
+                                                 p->G, p->G_pad);
+  }
   if (p->nls > 0)
     build_lr_codes_kernel<<<p->num_tiles * p->nls, 256, 0, s>>>(core_u, corr_a, p->lr_codes, p->V, p->rc, p->rr,
-                                                                 p->rcp, p->nls);
+                                                                 p->rcp, p->nls, p->sc4);
   build_row_scales_kernel<<<256, 256, 0, s>>>(p->rr > 0 ? corr_a_scale : nullptr, p->s_a, p->V, p->V_pad);
   if (p->lr > 0)
     build_lr_t_kernel<<<256, 256, 0, s>>>(p->q_v, p->q_b, p->lr_t, p->d, p->d_pad, p->rc, p->rr, p->rcp, p->lr);
@@ -120,6 +155,9 @@ cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, cons
 struct DequantArgs {
   const uint8_t *codes;
   const uint16_t *scales;
+  const uint8_t *scodes;
+  const uint16_t *s_row;
+  int sc4, G_pad2;
   const uint8_t *lr_codes;
   const uint16_t *s_a, *s_u, *s_v, *s_b;
   const int8_t *q_v, *q_b;
@@ -162,7 +200,14 @@ __global__ void debug_dequant_kernel(DequantArgs a, int comp, int64_t row0, int6
         uint32_t q[4];
         unpack_int4x8_biased(w, q);  // the decode kernel's operands: 136 + code
         const int grp = col / a.g;
-        v = (pair_half(q[i], h) - kInt4Bias) * fp16_bits_to_f32(a.scales[((int64_t)vt * a.G_pad + grp) * kTileRows + r]);
+        float sc;
+        if (a.sc4) {
+          const uint8_t b = a.scodes[((int64_t)vt * a.G_pad2 + (grp >> 1)) * kTileRows + r];
+          sc = fp16_bits_to_f32(a.s_row[row]) * (float)(((b >> (4 * (grp & 1))) & 15) + 1);
+        } else {
+          sc = fp16_bits_to_f32(a.scales[((int64_t)vt * a.G_pad + grp) * kTileRows + r]);
+        }
+        v = (pair_half(q[i], h) - kInt4Bias) * sc;
       } else {
         const int kk = comp == 1 ? col : a.rcp + col;
         const int ls = kk >> 4;
@@ -185,8 +230,9 @@ __global__ void debug_dequant_kernel(DequantArgs a, int comp, int64_t row0, int6
 
 cudaError_t launch_debug_dequant(const archead_pack *p, int comp, int64_t row0, int64_t nrows, float *out,
                                  cudaStream_t s) {
-  DequantArgs a{p->codes, p->scales, p->lr_codes, p->s_a, p->s_u, p->s_v, p->s_b, p->q_v, p->q_b,
-                p->d,     p->d_pad,  p->G_pad,    p->g,   p->rc,  p->rr,  p->rcp, p->nls};
+  DequantArgs a{p->codes, p->scales, p->scodes, p->s_row, p->sc4,  p->G_pad2, p->lr_codes, p->s_a,
+                p->s_u,   p->s_v,    p->s_b,    p->q_v,   p->q_b,  p->d,      p->d_pad,    p->G_pad,
+                p->g,     p->rc,     p->rr,     p->rcp,   p->nls};
   const int cols = comp == 0 ? p->d : ((comp == 1 || comp == 2) ? p->rc : p->rr);
   const int64_t total = nrows * cols;
   if (total == 0) return cudaSuccess;

@@ -123,6 +123,10 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
   DecodeParams dp{};
   dp.codes = pack->codes;
   dp.scales = pack->scales;
+  dp.scodes = pack->scodes;
+  dp.s_row = pack->s_row;
+  dp.sc4 = pack->sc4;
+  dp.G_pad2 = pack->G_pad2;
   dp.lr_codes = pack->lr_codes;
   dp.s_a = pack->s_a;
   dp.x = static_cast<const uint16_t *>(x);

@@ -45,7 +45,7 @@ def test_status_strings(lib):
 
 
 def _desc(**kw):
-    d = archead.archead_desc(vocab=100, hidden=256, core_rank=8, corr_rank=4, group_size=64, reserved=0)
+    d = archead.archead_desc(vocab=100, hidden=256, core_rank=8, corr_rank=4, group_size=64, format=0)
     dummy = ctypes.c_void_p(16)  # never dereferenced: the checks below fail first
     for name, _ in archead.archead_desc._fields_[6:]:
         setattr(d, name, dummy)
@@ -57,7 +57,7 @@ def _desc(**kw):
 @pytest.mark.parametrize("bad", [
     dict(vocab=0), dict(hidden=100), dict(hidden=32), dict(group_size=48), dict(group_size=16),
     dict(hidden=192, group_size=128), dict(core_rank=-1), dict(core_rank=257), dict(corr_rank=300),
-    dict(reserved=1), dict(res_codes=None), dict(res_scales=None), dict(core_u=None), dict(corr_b_scale=None),
+    dict(format=2), dict(format=-1), dict(format=1, res_row_scale=None), dict(res_codes=None), dict(res_scales=None), dict(core_u=None), dict(corr_b_scale=None),
 ])
 def test_pack_create_rejects_bad_desc(lib, bad):
     out = ctypes.c_void_p(1234)

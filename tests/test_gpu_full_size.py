@@ -1,5 +1,6 @@
-"""Full-size heads (the Qwen3-8B and Gemma-shaped configurations, the same
-seeded heads bench.py times) through the C ABI against the fp64 oracle:
+"""Full-size heads (the Qwen3-8B and Gemma-shaped configurations and the
+Qwen3-8B head in the paper's own packed format, the same seeded heads
+bench.py times) through the C ABI against the fp64 oracle:
 the whole vocabulary for decode token counts, sampled tokens for prefill
 (a token's logits depend on that token's hidden state only, so the oracle
 checks sampled rows exactly)."""
@@ -14,8 +15,8 @@ from tests import gpu_util as gu
 
 pytestmark = pytest.mark.gpu
 
-FULL = ("qwen3-8b", "gemma-4-e4b")
-PREFILL_M = {"qwen3-8b": 4096, "gemma-4-e4b": 2048}
+FULL = ("qwen3-8b", "gemma-4-e4b", "qwen3-8b-sc4")
+PREFILL_M = {"qwen3-8b": 4096, "gemma-4-e4b": 2048, "qwen3-8b-sc4": 4096}
 
 _state = {}
 

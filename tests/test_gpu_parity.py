@@ -25,6 +25,14 @@ SHAPES = {
     "corr_only": HeadShape(V=640, d=256, core_rank=0, corr_rank=32, group_size=64),
     "max_rank": HeadShape(V=384, d=256, core_rank=256, corr_rank=256, group_size=64),
     "one_row": HeadShape(V=1, d=64, core_rank=4, corr_rank=4, group_size=32),
+    # The paper's packed format (5-bit core left codes, 4-bit group-scale
+    # codes times a row scale), with its Qwen ranks and group size first.
+    "sc4": HeadShape(V=4096, d=512, core_rank=10, corr_rank=6, group_size=64, fmt="sc4"),
+    "sc4_ragged": HeadShape(V=1000, d=320, core_rank=10, corr_rank=6, group_size=64, fmt="sc4"),  # 5 groups
+    "sc4_g32": HeadShape(V=700, d=512, core_rank=24, corr_rank=40, group_size=32, fmt="sc4"),
+    "sc4_g128": HeadShape(V=513, d=512, core_rank=3, corr_rank=0, group_size=128, fmt="sc4"),
+    "sc4_g256": HeadShape(V=300, d=768, core_rank=13, corr_rank=5, group_size=256, fmt="sc4"),
+    "sc4_int4": HeadShape(V=640, d=256, core_rank=0, corr_rank=0, group_size=64, fmt="sc4"),
 }
 
 _packs = {}
@@ -104,7 +112,7 @@ def test_decode_hidden_state_range(M):
         gu.check_logits(got[m:m + 1], ref[m:m + 1], where=f"M={M} token {m}")
 
 
-@pytest.mark.parametrize("name", ["ragged", "tiny", "g32", "max_rank"])
+@pytest.mark.parametrize("name", ["ragged", "tiny", "g32", "max_rank", "sc4", "sc4_ragged", "sc4_g256", "sc4_int4"])
 @pytest.mark.parametrize("M", [17, 40, 133])
 def test_logits_many_tokens(name, M):
     pack, head = get(name)
@@ -117,7 +125,8 @@ def test_logits_many_tokens(name, M):
         gu.check_argmax(got, ref, where=f"{name} M={M} path={path}")
 
 
-@pytest.mark.parametrize("name", ["ragged", "tiny", "g32", "g256", "corr_only", "one_row", "max_rank"])
+@pytest.mark.parametrize("name", ["ragged", "tiny", "g32", "g256", "corr_only", "one_row", "max_rank", "sc4",
+                                  "sc4_g32"])
 @pytest.mark.parametrize("M", [1, 7, 16, 40])
 def test_greedy(name, M):
     pack, head = get(name)
@@ -129,7 +138,8 @@ def test_greedy(name, M):
         gu.check_greedy(idx, val, ref, where=f"{name} M={M} path={path}")
 
 
-@pytest.mark.parametrize("name", ["ragged", "tiny", "g32", "g256", "corr_only", "one_row"])
+@pytest.mark.parametrize("name", ["ragged", "tiny", "g32", "g256", "corr_only", "one_row", "sc4", "sc4_ragged",
+                                  "sc4_g128"])
 @pytest.mark.parametrize("M", [1, 5, 16, 33])
 def test_cross_entropy(name, M):
     pack, head = get(name)
@@ -191,7 +201,7 @@ def test_wait_timeout_is_reported_and_recoverable():
 
 
 def test_pack_bytes_follow_eq10():
-    for name in ("tiny", "group_int4", "core_only", "max_rank"):
+    for name in ("tiny", "group_int4", "core_only", "max_rank", "sc4", "sc4_ragged", "sc4_int4"):
         pack, head = get(name)
         assert archead.archead_pack_bytes(pack) == oracle.packed_bytes(SHAPES[name])
         assert archead.archead_device_bytes(pack) >= archead.archead_pack_bytes(pack)
