@@ -51,8 +51,8 @@ WORKLOADS = {
 
 
 KERNEL_SOURCES = {
-    "decode": ("decode.cu", "device.cuh", "internal.h"),
-    "prefill": ("prefill.cu", "device.cuh", "internal.h"),
+    "decode": ("decode.cu", "decode_sc4.cu", "decode_kernel.cuh", "device.cuh", "internal.h"),
+    "prefill": ("prefill.cu", "prefill_sc4.cu", "prefill_kernel.cuh", "device.cuh", "internal.h"),
 }
 
 

@@ -357,8 +357,14 @@ archead_status archead_pack_create(const archead_desc *desc, void *stream, arche
   p->G_pad2 = (p->G_pad + 1) / 2;
   p->num_tiles = (int)((V + kTileRows - 1) / kTileRows);
   p->V_pad = (int64_t)p->num_tiles * kTileRows;
-  p->rcp = (int)round_up(rc, 32);
-  p->rrp = (int)round_up(rr, 32);
+  // Extended rank axis: each branch padded to 16 columns (one k16 step), the
+  // sum to 32 (whole 64-wide k steps of the prefill's hi/lo operand).
+  p->rcp = (int)round_up(rc, 16);
+  p->rrp = (int)round_up(rr, 16);
+  if ((p->rcp + p->rrp) % 32 != 0) {
+    if (rr > 0) p->rrp += 16;
+    else p->rcp += 16;
+  }
   p->lr = p->rcp + p->rrp;
   p->nls = p->lr / 16;
   p->nls_core = p->rcp / 16;

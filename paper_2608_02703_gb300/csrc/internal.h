@@ -23,7 +23,8 @@
 //  into the low-rank codes below at pack time.
 //
 //  Low-rank codes: the extended rank axis kk in [0, LR) with LR = RCP + RRP,
-//  RCP = r_c rounded up to 32, RRP = r_r rounded up to 32: kk < RCP is
+//  RCP = r_c and RRP = r_r rounded up to 16, one of them raised by 16 when
+//  the sum is not a multiple of 32 (RRP if r_r > 0): kk < RCP is
 //  core_u[:, kk], kk >= RCP is corr_a[:, kk - RCP] (zero beyond the rank).
 //  Step ls (16 wide) of tile vt: [mi][lane][8 bytes], bytes 2i, 2i+1 = pair i
 //  (same row/column rule as above with 16*ls in place of the k16 offset),

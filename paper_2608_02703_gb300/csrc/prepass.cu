@@ -13,7 +13,8 @@
 //
 // Grid: (32 extended columns, 16 tokens, 256-wide split of d).  In a block,
 // warp w takes the 32-wide slice w of its split (a slice never straddles a
-// quantisation group, g >= 32), lane = column; a slice's partial sums are
+// quantisation group, g >= 32), lane = column (core or correction: RCP is a
+// multiple of 16, so a block may hold both); a slice's partial sums are
 // scaled by their group scale.  The eight warps' sums are added in a fixed
 // order and written per split; the last block of a (columns, tokens) pair to
 // finish adds the splits in split order and finalises (deterministic).
@@ -50,7 +51,7 @@ __global__ void __launch_bounds__(256) prepass_kernel(PrepassParams p) {
   const int k0 = blockIdx.z * kPreChunk;
   const int nsplit = gridDim.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const bool core = c0 < p.rcp;  // a 32-column block never straddles the core/correction boundary
+  const bool core = c0 + lane < p.rcp;  // a block may hold core and correction columns
   const int j = core ? c0 + lane : c0 + lane - p.rcp;
   const bool valid = core ? j < p.rc : j < p.rr;
   const int8_t *q = core ? p.q_v : p.q_b;
@@ -200,7 +201,8 @@ __global__ void __launch_bounds__(128) prepass_t_kernel(PrepassParams p, const u
   const int m0 = blockIdx.y * kPtTok;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gq = lane >> 2, cq = lane & 3;
-  const bool core = c0 < p.rcp;  // a 32-column block never straddles the core/correction boundary
+  // Eight-column slice n of the block is core (< RCP, a multiple of 16) or correction.
+  auto core_n = [&](int n) { return c0 + n * 8 < p.rcp; };
   const int nchunks = d_pad / kPtK;
 
   auto stage = [&](int kc, int buf) {
@@ -255,13 +257,15 @@ __global__ void __launch_bounds__(128) prepass_t_kernel(PrepassParams p, const u
         const uint16_t *br = xb + (n * 8 + gq) * kPtStride + kb;
         mma_bf16_16816(acc[n], a, *reinterpret_cast<const uint32_t *>(br), *reinterpret_cast<const uint32_t *>(br + 8));
       }
-      // End of a quantisation group of the correction factor: apply s_b.
+      // End of a quantisation group of the correction factor: apply s_b to
+      // the correction slices (core slices keep accumulating).
       const int kend = kc * kPtK + ks * 16 + 16;
-      if (!core && kend % p.g == 0) {
+      if (kend % p.g == 0) {
         const int grp = kend / p.g - 1;
-        if (grp < p.d / p.g) {
 #pragma unroll
-          for (int n = 0; n < 4; ++n) {
+        for (int n = 0; n < 4; ++n) {
+          if (core_n(n)) continue;
+          if (grp < p.d / p.g) {
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
               const int j = c0 - p.rcp + n * 8 + 2 * cq + h;
@@ -270,11 +274,9 @@ __global__ void __launch_bounds__(128) prepass_t_kernel(PrepassParams p, const u
               run[n][2 + h] = fmaf(sb, acc[n][2 + h], run[n][2 + h]);
             }
           }
-        }
-#pragma unroll
-        for (int n = 0; n < 4; ++n)
 #pragma unroll
           for (int i = 0; i < 4; ++i) acc[n][i] = 0.f;
+        }
       }
     }
   }
@@ -282,6 +284,7 @@ __global__ void __launch_bounds__(128) prepass_t_kernel(PrepassParams p, const u
   // t for (token, column) pairs of this lane, then the bf16 hi/lo split.
 #pragma unroll
   for (int n = 0; n < 4; ++n) {
+    const bool core = core_n(n);
 #pragma unroll
     for (int rh = 0; rh < 2; ++rh) {
       const int m = m0 + warp * 16 + gq + 8 * rh;
