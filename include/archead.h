@@ -70,7 +70,7 @@ typedef enum {
 } archead_format;
 
 typedef enum {
-  ARCHEAD_PATH_AUTO = 0,    /* decode kernel for M <= 16, prefill kernel above          */
+  ARCHEAD_PATH_AUTO = 0,    /* decode kernel for M <= 48, prefill kernel above          */
   ARCHEAD_PATH_DECODE = 1,  /* memory-bound decode kernel (tokens taken 16 at a time)   */
   ARCHEAD_PATH_PREFILL = 2  /* tensor-core prefill kernel                               */
 } archead_path;
