@@ -24,6 +24,8 @@ SHAPES = [
     HeadShape(V=1000, d=256, core_rank=16, corr_rank=8, group_size=64),
     HeadShape(V=4096, d=512, core_rank=64, corr_rank=16, group_size=64),
     HeadShape(V=700, d=320, core_rank=24, corr_rank=40, group_size=32),
+    # the paper's packed format (5-bit core codes, 4-bit group-scale codes)
+    HeadShape(V=1500, d=384, core_rank=10, corr_rank=6, group_size=64, fmt="sc4"),
 ]
 
 
@@ -45,7 +47,7 @@ def _run_noalloc(pack, x_bits, out_dtype):
     return y.float().cpu().numpy().astype(np.float64)
 
 
-@pytest.mark.parametrize("shape", SHAPES, ids=lambda s: f"V{s.V}_d{s.d}_g{s.group_size}")
+@pytest.mark.parametrize("shape", SHAPES, ids=lambda s: f"V{s.V}_d{s.d}_g{s.group_size}_{s.fmt}")
 @pytest.mark.parametrize("out_dtype", [archead.OUT_FP32, archead.OUT_BF16])
 def test_noalloc_matches_forward_on_two_calls_in_a_row(shape, out_dtype):
     head = make_head(shape, seed=zlib.crc32(repr(shape).encode()) % 1000)
