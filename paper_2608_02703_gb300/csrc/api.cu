@@ -4,7 +4,10 @@
 
 #include <algorithm>
 #include <cstring>
+#include <map>
+#include <mutex>
 #include <string>
+#include <utility>
 
 #include "device.cuh"
 #include "internal.h"
@@ -283,6 +286,20 @@ archead_status run_forward(archead_pack *p, const void *x, int64_t M, void *out,
 namespace archead {
 
 void set_last_error_message(const char *msg) { g_last_error = msg ? msg : ""; }
+
+cudaError_t opt_in_smem(const void *func, int bytes) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  static std::mutex mu;
+  static std::map<std::pair<const void *, int>, int> opted;  // (kernel, device) -> bytes
+  std::lock_guard<std::mutex> lock(mu);
+  int &have = opted[{func, dev}];
+  if (have >= bytes) return cudaSuccess;
+  e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) have = bytes;
+  return e;
+}
 
 void timer_begin(archead_pack *p, const char *name, cudaStream_t s, cudaEvent_t *ev0) {
   *ev0 = nullptr;

@@ -719,12 +719,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
 template <int NT, int SC, int GS, bool kSC4>
 static cudaError_t launch_t(const DecodeParams &dp, int grid, cudaStream_t s, const DecodePlan &pl, bool pdl) {
   auto kern = decode_kernel<NT, SC, GS, kSC4>;
-  static int smem_set = 0;  // largest dynamic shared memory opted in so far for this instance
-  if ((int)pl.total > smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)pl.total);
-    if (e != cudaSuccess) return e;
-    smem_set = (int)pl.total;
-  }
+  cudaError_t e = opt_in_smem(reinterpret_cast<const void *>(kern), (int)pl.total);
+  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kDecThreads);

@@ -175,6 +175,10 @@ cudaError_t launch_ce_finalize(const float2 *part, int num_parts, const float *t
                                int64_t V, int M, float *ce, int *err, cudaStream_t s);
 cudaError_t launch_wait_timeout_probe(int *err, int64_t budget, cudaStream_t s);
 
+// Opt `func` into `bytes` of dynamic shared memory on the current device:
+// once per kernel, device and size (the attribute is per device); thread-safe.
+cudaError_t opt_in_smem(const void *func, int bytes);
+
 // Message returned by archead_last_error() for this thread.
 void set_last_error_message(const char *msg);
 

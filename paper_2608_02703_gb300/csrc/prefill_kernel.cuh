@@ -604,28 +604,16 @@ cudaError_t launch_prefill_fmt(const archead_pack *pk, const void *x, int M, con
   const int tiles = p.num_vt * p.num_mt;
   const int grid = tiles < pk->sm_count ? tiles : pk->sm_count;
   if (out) {
-    static bool attr = false;
-    if (!attr) {
-      cudaError_t e = cudaFuncSetAttribute(prefill_kernel<0, kSC4>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPfSmem);
-      if (e != cudaSuccess) return e;
-      attr = true;
-    }
+    cudaError_t e = opt_in_smem(reinterpret_cast<const void *>(prefill_kernel<0, kSC4>), kPfSmem);
+    if (e != cudaSuccess) return e;
     prefill_kernel<0, kSC4><<<grid, kPfThreads, kPfSmem, s>>>(p);
   } else if (argmax) {
-    static bool attr = false;
-    if (!attr) {
-      cudaError_t e = cudaFuncSetAttribute(prefill_kernel<2, kSC4>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPfSmem);
-      if (e != cudaSuccess) return e;
-      attr = true;
-    }
+    cudaError_t e = opt_in_smem(reinterpret_cast<const void *>(prefill_kernel<2, kSC4>), kPfSmem);
+    if (e != cudaSuccess) return e;
     prefill_kernel<2, kSC4><<<grid, kPfThreads, kPfSmem, s>>>(p);
   } else {
-    static bool attr = false;
-    if (!attr) {
-      cudaError_t e = cudaFuncSetAttribute(prefill_kernel<1, kSC4>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPfSmem);
-      if (e != cudaSuccess) return e;
-      attr = true;
-    }
+    cudaError_t e = opt_in_smem(reinterpret_cast<const void *>(prefill_kernel<1, kSC4>), kPfSmem);
+    if (e != cudaSuccess) return e;
     prefill_kernel<1, kSC4><<<grid, kPfThreads, kPfSmem, s>>>(p);
   }
   return cudaGetLastError();

@@ -319,12 +319,8 @@ cudaError_t launch_prepass_t(const PrepassParams &pp, const uint16_t *lr_t, int 
   if (pp.lr == 0) return cudaSuccess;
   cudaEvent_t ev = nullptr;
   timer_begin(pk, "prepass", s, &ev);
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(prepass_t_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kPtSmem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  cudaError_t e = opt_in_smem(reinterpret_cast<const void *>(prepass_t_kernel), kPtSmem);
+  if (e != cudaSuccess) return e;
   dim3 grid(pp.lr / kPtCols, (pp.M + kPtTok - 1) / kPtTok);
   prepass_t_kernel<<<grid, 128, kPtSmem, s>>>(pp, lr_t, d_pad);
   timer_end(pk, "prepass", s, ev);
@@ -346,7 +342,7 @@ cudaError_t launch_prepass(const PrepassParams &pp, cudaStream_t s, archead_pack
   dim3 grid(pp.lr / kPreCols, (pp.M + kPreTok - 1) / kPreTok, (pp.d + kPreChunk - 1) / kPreChunk);
   const size_t smem = prepass_smem(pp.M);
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(prepass_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = opt_in_smem(reinterpret_cast<const void *>(prepass_kernel), (int)smem);
     if (e != cudaSuccess) return e;
   }
   prepass_kernel<<<grid, 256, smem, s>>>(pp);
