@@ -207,7 +207,7 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   for (int c = 0; c < f.nchunks; ++c) {
     dp.m0 = c * kDecodeMaxTokens;
     dp.M = (int)std::min<int64_t>(kDecodeMaxTokens, M - dp.m0);
-    dp.NT = dp.M > 8 ? 2 : 1;
+    dp.NT = decode_nt(p->d_pad, p->nls, p->g, dp.M);
     dp.ts = pp.ts + (size_t)c * p->nls * 256;
     cudaEvent_t ev = nullptr;
     timer_begin(p, "decode", s, &ev);

@@ -8,7 +8,16 @@ int decode_num_units(const archead_pack *p) { return (p->num_tiles + kDecTiles -
 
 int decode_parts_per_unit() { return kDecWarps; }
 
-bool decode_supported(int d_pad, int nls, int g) { return decode_plan(d_pad, nls, g, kDecodeMaxTokens).stages >= 2; }
+bool decode_supported(int d_pad, int nls, int g) { return decode_plan(d_pad, nls, g, kDecodeMaxTokens, 2).stages >= 2; }
+
+// One n-tile (x resident in shared memory as fp16) while that leaves a ring
+// of at least 96 KB; otherwise the two-tile instance, which streams x through
+// the ring (very wide heads: 8 tokens of d = 16384 would take 256 KB).
+int decode_nt(int d_pad, int nls, int g, int M) {
+  if (M > 8) return 2;
+  const DecodePlan pl = decode_plan(d_pad, nls, g, M, 1);
+  return pl.stages >= 2 && pl.xs_off >= (size_t)96 * 1024 ? 1 : 2;
+}
 
 extern template cudaError_t launch_decode_fmt<true>(const DecodeParams &, int, cudaStream_t, bool);
 template cudaError_t launch_decode_fmt<false>(const DecodeParams &, int, cudaStream_t, bool);

@@ -73,9 +73,8 @@ __host__ __device__ __forceinline__ int xs_row_elems(int d_pad) { return d_pad +
 // fragments, the per-group sums of x, and the barriers.  The total leaves
 // room for one pre-pass block on the same SM (programmatic dependent launch
 // overlaps the two grids) whenever the stage ring still holds 96 KB.
-static DecodePlan decode_plan(int d_pad, int nls, int g, int M) {
+static DecodePlan decode_plan(int d_pad, int nls, int g, int M, int nt) {
   DecodePlan pl{};
-  const int nt = M > 8 ? 2 : 1;
   const bool xs = streams_x(nt);
   pl.sc = stage_chunks(nt);
   const size_t stage_bytes = pl.sc == 2 ? (xs ? StageGeom<2, true>::kBytes : StageGeom<2, false>::kBytes)
@@ -750,10 +749,11 @@ static cudaError_t launch_g(const DecodeParams &dp, int grid, cudaStream_t s, co
 // so that the two sets compile in parallel).
 template <bool kSC4>
 cudaError_t launch_decode_fmt(const DecodeParams &dp, int grid, cudaStream_t s, bool pdl) {
-  const DecodePlan pl = decode_plan(dp.d_pad, dp.nls, dp.g, dp.M);
+  const DecodePlan pl = decode_plan(dp.d_pad, dp.nls, dp.g, dp.M, dp.NT);
   if (pl.stages < 2) return cudaErrorInvalidValue;
   static_assert(stage_chunks(1) >= 1 && stage_chunks(2) >= 1, "stage width");
-  if ((dp.NT == 1) != (dp.M <= 8) || pl.sc != stage_chunks(dp.NT)) return cudaErrorInvalidValue;
+  if ((dp.NT != 1 && dp.NT != 2) || (dp.NT == 1 && dp.M > 8) || pl.sc != stage_chunks(dp.NT))
+    return cudaErrorInvalidValue;
   if (dp.NT == 1) return launch_g<1, stage_chunks(1), kSC4>(dp, grid, s, pl, pdl);
   static_assert(streams_x(2) && !streams_x(1), "two n-tiles stream x");
   DecodeParams dx = dp;

@@ -164,6 +164,7 @@ bool make_tma_map_bf16(CUtensorMap *map, const void *base, int64_t rows, int64_t
 int decode_num_units(const archead_pack *p);
 int decode_parts_per_unit();
 bool decode_supported(int d_pad, int nls, int g);
+int decode_nt(int d_pad, int nls, int g, int M);  // n-tiles of 8 tokens of the instance to launch for M tokens
 cudaError_t launch_prefill(const archead_pack *pk, const void *x, int M, const uint16_t *T, void *out, int out_fp32,
                            bool argmax, const int32_t *targets, float2 *ce_part, float *ce_tlogit, cudaStream_t s);
 int prefill_parts_per_vt();

@@ -141,7 +141,7 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
   dp.nls_core = pack->nls_core;
   dp.M = (int)M;
   dp.m0 = 0;
-  dp.NT = M > 8 ? 2 : 1;
+  dp.NT = decode_nt(pack->d_pad, pack->nls, pack->g, (int)M);
   dp.out = logits;
   dp.out_fp32 = out_dtype == ARCHEAD_OUT_FP32;
   dp.M_total = (int)M;

@@ -154,6 +154,34 @@ def test_cross_entropy(name, M):
         assert np.all(err <= gu.CE_ABS), f"{name} M={M} path={path}: max|dCE|={err.max():.3e}"
 
 
+@pytest.mark.parametrize("shape", [
+    HeadShape(V=520, d=8192, core_rank=16, corr_rank=8, group_size=128),
+    HeadShape(V=300, d=6144, core_rank=10, corr_rank=6, group_size=64, fmt="sc4"),
+], ids=["d8192", "d6144_sc4"])
+def test_wide_head(shape):
+    """Heads so wide that eight tokens of x do not fit in shared memory next to
+    a deep enough ring: the decode path switches to its streamed-x instance
+    (at d = 8192 for M = 8); every path against the oracle.  One set of hidden
+    states (and its prefixes) keeps the Haar rotation of x to one draw."""
+    head = make_head(shape, seed=5)
+    pack = archead.archead_pack_create(head, shape)
+    try:
+        x = make_hidden(shape.d, 64, seed=5)
+        ref = oracle.logits(head, shape, x)
+        for M in (1, 5, 8, 16):
+            got = gu.forward(pack, x[:M], archead.OUT_FP32, archead.PATH_DECODE)
+            gu.check_logits(got, ref[:M], where=f"d={shape.d} decode M={M}")
+        got = gu.forward(pack, x, archead.OUT_FP32, archead.PATH_PREFILL)
+        gu.check_logits(got, ref, where=f"d={shape.d} prefill M=64")
+        t = make_targets(shape.V, 16, seed=5)
+        ce, st = gu.forward_ce(pack, x[:16], t)
+        assert st == archead.OK
+        ref_ce = oracle.cross_entropy(head, shape, x[:16], t)["ce"]
+        assert np.max(np.abs(ce - ref_ce)) <= gu.CE_ABS
+    finally:
+        pack.close()
+
+
 def test_ce_target_out_of_range():
     pack, head = get("ragged")
     shape = SHAPES["ragged"]
