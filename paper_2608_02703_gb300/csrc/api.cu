@@ -275,8 +275,11 @@ archead_status run_forward(archead_pack *p, const void *x, int64_t M, void *out,
   // AUTO: the decode kernel streams the head once per 16 tokens; a prefill
   // launch computes full 256-token tiles and costs about four decode passes
   // for M <= 256 (Qwen3-8B shape: ~360 us against ~95 us a pass), so up to
-  // three decode passes win.
-  const bool decode = path == ARCHEAD_PATH_DECODE || (path == ARCHEAD_PATH_AUTO && M <= 3 * kDecodeMaxTokens);
+  // three decode passes win.  Heads too wide for the decode kernel's shared
+  // memory plan (per-group sums of x for 16 tokens, e.g. d = 2^20 at g = 32)
+  // take the prefill kernel under AUTO.
+  const bool decode = path == ARCHEAD_PATH_DECODE ||
+                      (path == ARCHEAD_PATH_AUTO && M <= 3 * kDecodeMaxTokens && decode_supported(p->d_pad, p->nls, p->g));
   if (decode) return run_decode(p, x, M, out, out_fp32, targets, ce, amax_idx, amax_val, s);
   return run_prefill(p, x, M, out, out_fp32, targets, ce, amax_idx, amax_val, s);
 }

@@ -182,6 +182,33 @@ def test_wide_head(shape):
         pack.close()
 
 
+def test_very_wide_head_takes_prefill_under_auto():
+    """d = 65536 at g = 32: the decode kernel's per-group sums of x do not fit
+    its shared memory, so an explicit decode request is refused as
+    unsupported and AUTO runs the prefill kernel, for any M."""
+    import torch
+
+    shape = HeadShape(V=300, d=65536, core_rank=8, corr_rank=8, group_size=32)
+    head = make_head(shape, seed=6)
+    pack = archead.archead_pack_create(head, shape)
+    try:
+        rng = np.random.default_rng(6)
+        M = 3
+        # bf16 values of both signs with exponents 2^-7 .. 2^3 (no rotation: the
+        # Haar draw of make_hidden is a 65536 x 65536 QR).
+        x = ((rng.integers(0, 2, (M, shape.d)) << 15) | (rng.integers(120, 131, (M, shape.d)) << 7)
+             | rng.integers(0, 128, (M, shape.d))).astype(np.uint16)
+        ref = oracle.logits(head, shape, x)
+        got = gu.forward(pack, x, archead.OUT_FP32, archead.PATH_AUTO)
+        gu.check_logits(got, ref, where="d=65536 auto")
+        y = torch.empty((M, shape.V), dtype=torch.float32, device="cuda")
+        with pytest.raises(archead.ArcheadError) as ei:
+            archead.archead_forward_path(pack, gu.to_dev(x), M, y, archead.OUT_FP32, archead.PATH_DECODE)
+        assert ei.value.status == archead.ERR_UNSUPPORTED
+    finally:
+        pack.close()
+
+
 def test_ce_target_out_of_range():
     pack, head = get("ragged")
     shape = SHAPES["ragged"]
