@@ -84,3 +84,41 @@ def test_null_pack_calls(lib):
     assert lib.archead_pack_bytes(None) == -1
     assert lib.archead_device_bytes(None) == -1
     lib.archead_destroy(None)
+
+
+C_CLIENT = r"""
+#include <stdio.h>
+#include <string.h>
+#include "archead.h"
+
+/* A plain C client: the header must compile as C11 and the library must be
+   callable without C++ (argument checks only; no device is needed). */
+int main(void) {
+  archead_desc d;
+  archead_pack *pack = (archead_pack *)1;
+  memset(&d, 0, sizeof d);
+  d.vocab = 100; d.hidden = 256; d.core_rank = 8; d.corr_rank = 4; d.group_size = 64;
+  d.format = ARCHEAD_FORMAT_SC4;  /* res_row_scale left NULL: rejected */
+  if (archead_pack_create(&d, NULL, &pack) != ARCHEAD_ERR_INVALID_ARG || pack != NULL) return 1;
+  if (archead_forward(NULL, NULL, 1, NULL, ARCHEAD_OUT_BF16, NULL) != ARCHEAD_ERR_INVALID_ARG) return 2;
+  if (strcmp(archead_status_string(ARCHEAD_ERR_UNSUPPORTED), "ARCHEAD_ERR_UNSUPPORTED") != 0) return 3;
+  if (archead_pack_bytes(NULL) != -1) return 4;
+  archead_destroy(NULL);
+  printf("c client ok\n");
+  return 0;
+}
+"""
+
+
+def test_plain_c_client_compiles_links_and_runs(lib, tmp_path):
+    import subprocess
+
+    src = tmp_path / "client.c"
+    src.write_text(C_CLIENT)
+    exe = tmp_path / "client"
+    libdir = os.path.dirname(archead.library_path())
+    subprocess.run(["gcc", "-std=c11", "-Wall", "-Werror", "-pedantic", f"-I{INCLUDE}", str(src), "-o", str(exe),
+                    f"-L{libdir}", "-larchead", f"-Wl,-rpath,{libdir}"], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert out.returncode == 0, out.stdout + out.stderr
+    assert "c client ok" in out.stdout
