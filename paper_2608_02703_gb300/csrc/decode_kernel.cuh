@@ -133,6 +133,12 @@ __device__ __forceinline__ float scale_mult(uint32_t b, int sh) {
   return __uint_as_float(0x4B000000u | ((b >> sh) & 15u)) - 8388607.0f;
 }
 
+// (q + 1) / 16 the same way: the code as the low mantissa bits of 2^19
+// (unit 1/16), minus 2^19 - 1/16 (exact).
+__device__ __forceinline__ float scale_mult_16th(uint32_t b, int sh) {
+  return __uint_as_float(0x49000000u | ((b >> sh) & 15u)) - 524287.9375f;
+}
+
 // NT: n-tiles of 8 tokens; SC: 64-wide chunks per stage; GS: 16-wide k steps per group.
 template <int NT, int SC, int GS, bool kSC4>
 __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_constant__ DecodeParams p, int stages,
@@ -408,7 +414,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
 #pragma unroll
             for (int mt = 0; mt < kDecMT; ++mt) {
               s_lo[gi][mt] = scale_mult(sc8[br * kTileRows + mt * 16], sh);
-              s_hi[gi][mt] = scale_mult(sc8[br * kTileRows + mt * 16 + 8], sh) * (kF16 ? 0.0625f : 1.f);
+              const uint32_t bh = sc8[br * kTileRows + mt * 16 + 8];
+              s_hi[gi][mt] = kF16 ? scale_mult_16th(bh, sh) : scale_mult(bh, sh);  // fp16 operands: x16 rows
             }
           }
         } else {
