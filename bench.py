@@ -46,6 +46,8 @@ WORKLOADS = {
     "qwen3-8b-sc4-prefill": ("qwen3-8b-sc4", 4096, "logits"),
     "gemma-4-e4b-decode": ("gemma-4-e4b", 1, "logits"),
     "gemma-4-e4b-prefill": ("gemma-4-e4b", 2048, "logits"),
+    "gemma-4-e4b-decode": ("gemma-4-e4b", 1, "logits"),
+    "gemma-4-e4b-prefill": ("gemma-4-e4b", 2048, "logits"),
     "tiny": ("tiny", 4, "logits"),
 }
 
@@ -397,9 +399,23 @@ def run_ours(args, rank, world, local_rank):
     pack.close()
     if not args.no_extras and args.workload == "qwen3-8b-decode":
         result["sc4"] = sc4_block(peaks, world, local_rank)
+        result["gemma"] = gemma_block(peaks, world, local_rank)
     if rank == 0 and not args.no_cpu_baseline and world == 1:
         result["cpu_baseline"] = cpu_baseline(wl, x_np, M, budget_s=args.cpu_budget)
     return result
+
+
+def gemma_block(peaks, world, local_rank):
+    """The Gemma-4-E4B-shaped head (V=262144, d=2560, r_c=128, r_r=32, g=128):
+    decode M=1 and 8, prefill M=2048 (logits and fused CE)."""
+    wl = Workload("gemma-4-e4b")
+    pack = wl.open()
+    res = {"workload": "gemma-4-e4b head (V=262144, d=2560, r_c=128, r_r=32, g=128)",
+           "packed_bytes": packed_bytes(wl.shape),
+           "decode_sweep": decode_sweep(pack, wl.shape, peaks, world, local_rank, Ms=(1, 8)),
+           "prefill": prefill_block(pack, wl.shape, peaks, world, local_rank, M=2048)}
+    pack.close()
+    return res
 
 
 def sc4_block(peaks, world, local_rank):
@@ -438,13 +454,12 @@ def decode_sweep(pack, shape, peaks, world, local_rank, Ms=(1, 2, 4, 8, 16)):
     return out
 
 
-def prefill_block(pack, shape, peaks, world, local_rank):
+def prefill_block(pack, shape, peaks, world, local_rank, M=4096):
     import torch
 
     from paper_2608_02703_gb300 import archead
     from synth import make_hidden, make_targets
 
-    M = 4096
     x = torch.from_numpy(make_hidden(shape.d, M, seed=3, n_outliers=shape.n_outliers).view(np.int16)).cuda()
     y = torch.empty((M, shape.V), dtype=torch.bfloat16, device="cuda")
     tgt = torch.from_numpy(make_targets(shape.V, M, seed=3)).cuda()
