@@ -14,6 +14,7 @@ import zlib
 import numpy as np
 import pytest
 
+import oracle
 from paper_2608_02703_gb300 import archead
 from synth import HeadShape, make_head, make_hidden
 from tests import gpu_util as gu
@@ -95,5 +96,37 @@ def test_noalloc_rejects_heads_needing_more_scratch():
             archead.archead_forward_decode_noalloc(pack, x, 1, y, archead.OUT_FP32)
         assert exc.value.status == archead.ERR_UNSUPPORTED
         assert "512 KiB" in str(exc.value)
+    finally:
+        pack.close()
+
+
+def test_noalloc_forward_replays_as_a_cuda_graph():
+    """The allocation-free decode captured once into a CUDA graph (pre-pass and
+    decode grids with their programmatic dependency) and replayed on new
+    hidden states written into the captured input buffer."""
+    import torch
+
+    shape = SHAPES[1]
+    head = make_head(shape, seed=7)
+    pack = archead.archead_pack_create(head, shape)
+    try:
+        M = 5
+        xd = torch.zeros((M, shape.d), dtype=torch.int16, device="cuda")
+        y = torch.zeros((M, shape.V), dtype=torch.float32, device="cuda")
+        # First call outside the capture: it looks up the scratch array's
+        # device address and opts the kernels into their shared memory.
+        archead.archead_forward_decode_noalloc(pack, xd, M, y, archead.OUT_FP32)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            archead.archead_forward_decode_noalloc(pack, xd, M, y, archead.OUT_FP32)
+        for seed in (8, 9):
+            x = make_hidden(shape.d, M, seed=seed)
+            xd.copy_(torch.from_numpy(x.view(np.int16)))
+            g.replay()
+            torch.cuda.synchronize()
+            assert archead.archead_sync_status(pack) == archead.OK
+            got = y.cpu().numpy().astype(np.float64)
+            gu.check_logits(got, oracle.logits(head, shape, x), where=f"graph replay seed={seed}")
     finally:
         pack.close()
