@@ -1,0 +1,39 @@
+"""bench.py's algorithmic byte and flop accounting and its use of the
+committed traffic captures (host logic, CPU only)."""
+
+import json
+
+import bench
+import oracle
+from synth import SHAPES, HeadShape
+
+
+def test_packed_bytes_match_the_oracle_eq10():
+    for name in ("tiny", "qwen3-8b", "gemma-4-e4b", "tiny-sc4", "qwen3-8b-sc4"):
+        assert bench.packed_bytes(SHAPES[name]) == oracle.packed_bytes(SHAPES[name]), name
+    odd = HeadShape(V=333, d=320, core_rank=13, corr_rank=0, group_size=64, fmt="sc4")
+    assert bench.packed_bytes(odd) == oracle.packed_bytes(odd)
+
+
+def test_streamed_bytes_are_the_vocabulary_side_of_the_pack():
+    s = SHAPES["qwen3-8b"]
+    d_side = s.d * s.core_rank + 2 * 2 * s.core_rank + s.d * s.corr_rank + (s.d // s.group_size) * s.corr_rank * 2
+    assert bench.packed_vocab_bytes(s) + d_side == bench.packed_bytes(s)
+    assert bench.kernel_bytes(s, 1, "logits") == bench.packed_vocab_bytes(s) + 2 * s.d + 2 * s.V
+    assert bench.call_flops(s, 4096) == 2 * 4096 * s.V * s.d + 2 * 4096 * (s.V + s.d) * (s.core_rank + s.corr_rank)
+
+
+def test_traffic_is_used_only_for_the_sources_it_was_captured_with(tmp_path, monkeypatch):
+    """A capture counts only for its kernel, workload and M, and only while the
+    kernel's sources hash to the ones it was taken with (else null)."""
+    table = {"decode/qwen3-8b-decode/M=1": {"dram_bytes_per_launch": 123, "sources_sha256": bench.kernel_source_hash("decode")},
+             "prefill/qwen3-8b-prefill/M=1024": {"dram_bytes_per_launch": 456, "sources_sha256": "0" * 64}}
+    (tmp_path / "profiles").mkdir()
+    (tmp_path / "profiles" / "traffic.json").write_text(json.dumps(table))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    monkeypatch.setattr(bench, "kernel_source_hash", lambda k: table["decode/qwen3-8b-decode/M=1"]["sources_sha256"]
+                        if k == "decode" else "1" * 64)
+    assert bench.captured_traffic("decode", "qwen3-8b-decode", 1) == 123
+    assert bench.captured_traffic("decode", "qwen3-8b-decode", 16) is None      # no capture at this M
+    assert bench.captured_traffic("prefill", "qwen3-8b-prefill", 1024) is None  # sources changed since
+
