@@ -7,8 +7,10 @@ stream with group promotion, low-rank epilogue, logits store -- over one batch
 of seeded synthetic hidden states already resident in device memory.  The
 default workload is the Qwen3-8B-shaped head (V=151936, d=4096, r_c=128,
 r_r=32, g=128) at M=1 token (decode); the same line also carries the decode
-sweep M=2..16, the M=4096 prefill (logits and fused cross entropy) and a dense
-BF16 cuBLAS head on the same shapes.
+sweep M=2..16, the M=4096 prefill (logits and fused cross entropy), a dense
+BF16 cuBLAS head on the same shapes, the batch sweep M=1..8192 through both
+kernels, the same head in the paper's own packed format, and the
+Gemma-4-E4B-shaped head.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -44,8 +46,6 @@ WORKLOADS = {
     # the same head shape in the paper's own packed format (r_c = 10, r_r = 6, g = 64)
     "qwen3-8b-sc4-decode": ("qwen3-8b-sc4", 1, "logits"),
     "qwen3-8b-sc4-prefill": ("qwen3-8b-sc4", 4096, "logits"),
-    "gemma-4-e4b-decode": ("gemma-4-e4b", 1, "logits"),
-    "gemma-4-e4b-prefill": ("gemma-4-e4b", 2048, "logits"),
     "gemma-4-e4b-decode": ("gemma-4-e4b", 1, "logits"),
     "gemma-4-e4b-prefill": ("gemma-4-e4b", 2048, "logits"),
     "tiny": ("tiny", 4, "logits"),
