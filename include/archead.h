@@ -70,8 +70,10 @@ typedef enum {
 } archead_format;
 
 typedef enum {
-  ARCHEAD_PATH_AUTO = 0,    /* decode kernel for M <= 48, prefill kernel above          */
-  ARCHEAD_PATH_DECODE = 1,  /* memory-bound decode kernel (tokens taken 16 at a time)   */
+  ARCHEAD_PATH_AUTO = 0,    /* decode kernel for M <= 48, prefill kernel above (and for
+                               heads too wide for the decode kernel's shared memory)  */
+  ARCHEAD_PATH_DECODE = 1,  /* memory-bound decode kernel (tokens taken 16 at a time);
+                               ARCHEAD_ERR_UNSUPPORTED for heads too wide for it     */
   ARCHEAD_PATH_PREFILL = 2  /* tensor-core prefill kernel                               */
 } archead_path;
 
