@@ -195,6 +195,49 @@ ARCHEAD_API archead_status archead_forward_argmax_path(archead_pack *pack, const
                                                        float *value, archead_path path, void *stream);
 
 /*
+ * Vocabulary-parallel evaluation.  The forward is row-separable (paper,
+ * Section 3.2, Eq. 7: every logit y[m][n] involves only row n of the
+ * V-indexed components -- residual codes and scales, core_u, corr_a and its
+ * row scales -- and the d-side factors core_v, corr_b, which every shard
+ * holds whole).  A head can therefore be cut into P contiguous blocks of
+ * vocabulary rows, one pack per block (shard p holds global rows
+ * [row0_p, row0_p + V_p) as its rows 0..V_p-1), typically one per GPU:
+ * logits need no exchange (each shard writes its own columns), cross entropy
+ * and greedy output need one small exchange per token, made by the caller
+ * (an all-gather over its process group, for example), followed by one of
+ * the combines below.
+ *
+ * archead_forward_lse_partial: for each token m, over this shard's rows,
+ *   parts[3m]     = max_n y[m][n]
+ *   parts[3m + 1] = sum_n exp(y[m][n] - parts[3m])
+ *   parts[3m + 2] = y[m][targets[m] - row0] if row0 <= targets[m] < row0 + V
+ *                   of this pack, else -inf (another shard owns the target).
+ *   x device bf16 [M][d]; targets device int32 [M] (GLOBAL rows);
+ *   parts device fp32 [M][3], 16-byte aligned (caller-owned).
+ *   row0 is this shard's first global row (row0 + V < 2^31).
+ *
+ * archead_lse_combine: parts device fp32 [num_shards][M][3], the shards'
+ * partials in shard order; ce device fp32 [M]:
+ *   ce[m] = max + log(sum) - y[m][t_m]   (merged over the shards in order),
+ * NaN where no shard (or more than one) reports the target.  Uses the
+ * current device; deterministic.
+ *
+ * archead_argmax_combine: values fp32 [num_shards][M] and indices int32
+ * [num_shards][M] from each shard's archead_forward_argmax (shard-local
+ * rows), row0 int32 [num_shards] the shards' first global rows, all device
+ * memory; writes index[m] = the global row of the largest logit over all
+ * shards (the lowest row on ties, as argmax) and, if value != NULL, that
+ * logit.  Uses the current device; deterministic.
+ */
+ARCHEAD_API archead_status archead_forward_lse_partial(archead_pack *pack, const void *x, int64_t M,
+                                                       const int32_t *targets, int64_t row0, float *parts,
+                                                       archead_path path, void *stream);
+ARCHEAD_API archead_status archead_lse_combine(const float *parts, int num_shards, int64_t M, float *ce, void *stream);
+ARCHEAD_API archead_status archead_argmax_combine(const float *values, const int32_t *indices, const int32_t *row0,
+                                                  int num_shards, int64_t M, int32_t *index, float *value,
+                                                  void *stream);
+
+/*
  * End-to-end call with HOST buffers: copies x (host, bf16 [M][d]) to the
  * device, runs archead_forward, copies the logits back to logits_host
  * ([M][V], bf16 or fp32) and waits for the stream.  Pinned host memory
@@ -258,10 +301,13 @@ ARCHEAD_API archead_status archead_debug_wait_timeout(archead_pack *pack, void *
  * one fixed 512 KiB array compiled into the library, which every device that
  * loads the library holds until the process exits.
  *   x       device, bf16 [M][d];  logits device, [M][V] (bf16 or fp32), as archead_forward.
- * The first call on a device looks up that array's device address; make that
- * first call before any stream capture.  All calls on a device share the
- * array: calls whose work overlaps on the GPU (other streams, other packs at
- * the same time) race.  Returns ARCHEAD_ERR_UNSUPPORTED (see
+ * The first call with a pack (at any M <= 16) looks up that array's device
+ * address on the pack's device and prepares every decode kernel the pack can
+ * use; make that first call before any stream capture.  The address is kept
+ * for the life of the process, so calls after a cudaDeviceReset of that
+ * device are not supported.  All calls on a device share the array: calls
+ * whose work overlaps on the GPU (other streams, other packs at the same
+ * time) race.  Returns ARCHEAD_ERR_UNSUPPORTED (see
  * archead_last_error) when M > 16 or the head needs more than 512 KiB of
  * scratch (pre-pass partial sums: 2 KB per 32 rank columns per 256 of d, plus
  * 1 KB per 16 rank columns; 174 KB for d=4096, r_c+r_r=160).

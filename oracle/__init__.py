@@ -251,3 +251,40 @@ def dense_bf16_bytes(V: int, d: int) -> int:
 
 def threads() -> int:
     return int(_load().oracle_threads())
+
+
+# ---------------------------------------------------------------------------
+# Vocabulary shards (the forward is row-separable, paper Section 3.2, Eq. 7).
+# ---------------------------------------------------------------------------
+def lse_partial(head, shape, x_bits: np.ndarray, targets: np.ndarray, row0: int, nrows: int) -> np.ndarray:
+    """fp64 (max, sum of exp(y - max), target logit or -inf) per token over
+    global rows [row0, row0 + nrows) of the head: [M, 3]."""
+    y = logits(head, shape, x_bits, row0=row0, nrows=nrows)
+    mx = y.max(axis=1)
+    s = np.exp(y - mx[:, None]).sum(axis=1)
+    t = np.asarray(targets, dtype=np.int64) - row0
+    mine = (t >= 0) & (t < nrows)
+    tl = np.where(mine, y[np.arange(y.shape[0]), np.clip(t, 0, nrows - 1)], -np.inf)
+    return np.stack([mx, s, tl], axis=1)
+
+
+def lse_combine(parts: np.ndarray) -> np.ndarray:
+    """CE per token from shard partials [P, M, 3] (shard order): the log-sum-
+    exp of the union of the shards' rows minus the one reported target logit;
+    NaN where the number of shards reporting the target is not one."""
+    parts = np.asarray(parts, dtype=np.float64)
+    mx = parts[:, :, 0].max(axis=0)
+    s = (parts[:, :, 1] * np.exp(parts[:, :, 0] - mx[None, :])).sum(axis=0)
+    owners = np.isfinite(parts[:, :, 2]).sum(axis=0)
+    t = np.where(np.isfinite(parts[:, :, 2]), parts[:, :, 2], 0.0).sum(axis=0)
+    return np.where(owners == 1, mx + np.log(s) - t, np.nan)
+
+
+def argmax_combine(values: np.ndarray, indices: np.ndarray, row0: np.ndarray):
+    """Greedy output over shards: the largest value, the lowest global row
+    (local index + the shard's row0) on ties.  values, indices [P, M]."""
+    values = np.asarray(values, dtype=np.float64)
+    glob = np.asarray(indices, dtype=np.int64) + np.asarray(row0, dtype=np.int64).reshape(-1, 1)
+    best = values.max(axis=0)
+    cand = np.where(values == best[None, :], glob, np.iinfo(np.int64).max)
+    return cand.min(axis=0), best

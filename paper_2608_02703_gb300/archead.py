@@ -43,6 +43,7 @@ EXPORTED = (
     "archead_debug_dequant", "archead_sync_status", "archead_set_wait_budget", "archead_debug_wait_timeout",
     "archead_profile_enable", "archead_profile_read", "archead_status_string", "archead_last_error",
     "archead_forward_decode_noalloc", "archead_forward_argmax", "archead_forward_argmax_path",
+    "archead_forward_lse_partial", "archead_lse_combine", "archead_argmax_combine",
 )
 
 
@@ -101,6 +102,9 @@ def load() -> ctypes.CDLL:
         "archead_forward_decode_noalloc": (i32, [vp, vp, i64, vp, i32, vp]),
         "archead_forward_argmax": (i32, [vp, vp, i64, vp, vp, vp]),
         "archead_forward_argmax_path": (i32, [vp, vp, i64, vp, vp, i32, vp]),
+        "archead_forward_lse_partial": (i32, [vp, vp, i64, vp, i64, vp, i32, vp]),
+        "archead_lse_combine": (i32, [vp, i32, i64, vp, vp]),
+        "archead_argmax_combine": (i32, [vp, vp, vp, i32, i64, vp, vp, vp]),
         "archead_pack_bytes": (i64, [vp]),
         "archead_device_bytes": (i64, [vp]),
         "archead_debug_dequant": (i32, [vp, i32, i64, i64, vp, vp]),
@@ -237,6 +241,25 @@ def archead_forward_decode_noalloc(pack: Pack, x, M: int, logits, out_dtype: int
     """archead_forward for M <= 16 without any device allocation (fixed 512 KiB scratch array in the library)."""
     _check(load().archead_forward_decode_noalloc(pack.handle, _ptr(x), M, _ptr(logits), out_dtype,
                                                  _stream_ptr(stream)), "archead_forward_decode_noalloc")
+
+
+def archead_forward_lse_partial(pack: Pack, x, M: int, targets, row0: int, parts, path: int = PATH_AUTO,
+                                stream=None) -> None:
+    """Per-token (max, sum of exp, target logit or -inf) over this shard's rows (fp32 [M][3])."""
+    _check(load().archead_forward_lse_partial(pack.handle, _ptr(x), M, _ptr(targets), row0, _ptr(parts), path,
+                                              _stream_ptr(stream)), "archead_forward_lse_partial")
+
+
+def archead_lse_combine(parts, num_shards: int, M: int, ce, stream=None) -> None:
+    """Cross entropy from the shards' partials (fp32 [num_shards][M][3], shard order)."""
+    _check(load().archead_lse_combine(_ptr(parts), num_shards, M, _ptr(ce), _stream_ptr(stream)),
+           "archead_lse_combine")
+
+
+def archead_argmax_combine(values, indices, row0, num_shards: int, M: int, index, value=None, stream=None) -> None:
+    """Greedy output from the shards' (value, local index) and their first global rows."""
+    _check(load().archead_argmax_combine(_ptr(values), _ptr(indices), _ptr(row0), num_shards, M, _ptr(index),
+                                         _ptr(value), _stream_ptr(stream)), "archead_argmax_combine")
 
 
 def archead_pack_bytes(pack: Pack) -> int:

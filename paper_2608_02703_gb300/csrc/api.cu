@@ -140,29 +140,11 @@ archead_status check_forward_args(archead_pack *p, const void *x, int64_t M, con
   return ARCHEAD_OK;
 }
 
-PrepassParams prepass_params(archead_pack *p, const void *x, int64_t M) {
-  PrepassParams pp{};
-  pp.x = static_cast<const uint16_t *>(x);
-  pp.q_v = p->q_v;
-  pp.q_b = p->q_b;
-  pp.s_b = p->s_b;
-  pp.s_u = p->s_u;
-  pp.s_v = p->s_v;
-  pp.M = (int)M;
-  pp.d = p->d;
-  pp.g = p->g;
-  pp.rc = p->rc;
-  pp.rr = p->rr;
-  pp.rcp = p->rcp;
-  pp.rrp = p->rrp;
-  pp.lr = p->lr;
-  return pp;
-}
-
 // Decode path over M tokens, 16 at a time.  out == nullptr selects CE mode,
 // or greedy mode when amax_idx is given.
 archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
-                          const int32_t *targets, float *ce, int32_t *amax_idx, float *amax_val, cudaStream_t s) {
+                          const int32_t *targets, float *ce, int32_t *amax_idx, float *amax_val, int row0,
+                          float *parts3, cudaStream_t s) {
   if (!decode_supported(p->d_pad, p->nls, p->g)) return ARCHEAD_ERR_UNSUPPORTED;
   const bool ce_mode = out == nullptr;
   const bool greedy = amax_idx != nullptr;
@@ -176,38 +158,19 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   pp.T = nullptr;
   AH_CUDA(launch_prepass(pp, s, p));
 
-  DecodeParams dp{};
-  dp.codes = p->codes;
-  dp.scales = p->scales;
-  dp.scodes = p->scodes;
-  dp.s_row = p->s_row;
-  dp.sc4 = p->sc4;
-  dp.G_pad2 = p->G_pad2;
-  dp.lr_codes = p->lr_codes;
-  dp.s_a = p->s_a;
-  dp.x = static_cast<const uint16_t *>(x);
-  dp.V = p->V;
-  dp.num_tiles = p->num_tiles;
-  dp.d = p->d;
-  dp.d_pad = p->d_pad;
-  dp.G_pad = p->G_pad;
-  dp.g = p->g;
-  dp.nls = p->nls;
-  dp.nls_core = p->nls_core;
+  DecodeParams dp = decode_params(p, x, M);
   dp.out = out;
   dp.out_fp32 = out_fp32;
   dp.targets = targets;
+  dp.row0 = row0;
   dp.argmax = greedy;
   dp.ce_part = ce_mode ? at<float2>(p->ws, f.ce_part_off) : nullptr;
   dp.ce_tlogit = ce_mode ? at<float>(p->ws, f.tlogit_off) : nullptr;
-  dp.M_total = (int)M;
-  dp.err = p->err;
-  dp.wait_budget = p->wait_budget;
   const int grid = std::min(decode_num_units(p), p->sm_count);
   for (int c = 0; c < f.nchunks; ++c) {
     dp.m0 = c * kDecodeMaxTokens;
     dp.M = (int)std::min<int64_t>(kDecodeMaxTokens, M - dp.m0);
-    dp.NT = decode_nt(p->d_pad, p->nls, p->g, dp.M);
+    dp.variant = decode_variant(p->d_pad, p->nls, p->g, dp.M);
     dp.ts = pp.ts + (size_t)c * p->nls * 256;
     cudaEvent_t ev = nullptr;
     timer_begin(p, "decode", s, &ev);
@@ -221,8 +184,10 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
     cudaEvent_t ev = nullptr;
     timer_begin(p, "ce_finalize", s, &ev);
     const int parts = decode_num_units(p) * decode_parts_per_unit();
-    cudaError_t e = greedy ? launch_argmax_finalize(dp.ce_part, parts, (int)M, amax_idx, amax_val, s)
-                           : launch_ce_finalize(dp.ce_part, parts, dp.ce_tlogit, targets, p->V, (int)M, ce, p->err, s);
+    cudaError_t e =
+        greedy   ? launch_argmax_finalize(dp.ce_part, parts, (int)M, amax_idx, amax_val, s)
+        : parts3 ? launch_lse_partial_finalize(dp.ce_part, parts, dp.ce_tlogit, targets, row0, p->V, (int)M, parts3, s)
+                 : launch_ce_finalize(dp.ce_part, parts, dp.ce_tlogit, targets, p->V, (int)M, ce, p->err, s);
     timer_end(p, "ce_finalize", s, ev);
     if (e != cudaSuccess) return cuda_status(e);
   }
@@ -233,7 +198,8 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
 // tensor-core kernel.  out == nullptr selects CE mode, or greedy mode when
 // amax_idx is given.
 archead_status run_prefill(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
-                           const int32_t *targets, float *ce, int32_t *amax_idx, float *amax_val, cudaStream_t s) {
+                           const int32_t *targets, float *ce, int32_t *amax_idx, float *amax_val, int row0,
+                           float *parts3, cudaStream_t s) {
   const bool ce_mode = out == nullptr;
   const bool greedy = amax_idx != nullptr;
   Carve c;
@@ -252,14 +218,15 @@ archead_status run_prefill(archead_pack *p, const void *x, int64_t M, void *out,
   float *tlogit = ce_mode ? at<float>(p->ws, tlogit_off) : nullptr;
   cudaEvent_t ev = nullptr;
   timer_begin(p, "prefill", s, &ev);
-  cudaError_t e = launch_prefill(p, x, (int)M, pp.T, out, out_fp32, greedy, targets, ce_part, tlogit, s);
+  cudaError_t e = launch_prefill(p, x, (int)M, pp.T, out, out_fp32, greedy, targets, row0, ce_part, tlogit, s);
   timer_end(p, "prefill", s, ev);
   if (e != cudaSuccess) return cuda_status(e);
   if (ce_mode) {
     timer_begin(p, "ce_finalize", s, &ev);
     const int parts = p->num_tiles * prefill_parts_per_vt();
-    e = greedy ? launch_argmax_finalize(ce_part, parts, (int)M, amax_idx, amax_val, s)
-               : launch_ce_finalize(ce_part, parts, tlogit, targets, p->V, (int)M, ce, p->err, s);
+    e = greedy   ? launch_argmax_finalize(ce_part, parts, (int)M, amax_idx, amax_val, s)
+        : parts3 ? launch_lse_partial_finalize(ce_part, parts, tlogit, targets, row0, p->V, (int)M, parts3, s)
+                 : launch_ce_finalize(ce_part, parts, tlogit, targets, p->V, (int)M, ce, p->err, s);
     timer_end(p, "ce_finalize", s, ev);
     if (e != cudaSuccess) return cuda_status(e);
   }
@@ -268,7 +235,8 @@ archead_status run_prefill(archead_pack *p, const void *x, int64_t M, void *out,
 
 archead_status run_forward(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
                            const int32_t *targets, float *ce, archead_path path, cudaStream_t s,
-                           int32_t *amax_idx = nullptr, float *amax_val = nullptr) {
+                           int32_t *amax_idx = nullptr, float *amax_val = nullptr, int row0 = 0,
+                           float *parts3 = nullptr) {
   if (path != ARCHEAD_PATH_AUTO && path != ARCHEAD_PATH_DECODE && path != ARCHEAD_PATH_PREFILL)
     return ARCHEAD_ERR_INVALID_ARG;
   AH_CUDA(cudaSetDevice(p->device));
@@ -280,8 +248,8 @@ archead_status run_forward(archead_pack *p, const void *x, int64_t M, void *out,
   // take the prefill kernel under AUTO.
   const bool decode = path == ARCHEAD_PATH_DECODE ||
                       (path == ARCHEAD_PATH_AUTO && M <= 3 * kDecodeMaxTokens && decode_supported(p->d_pad, p->nls, p->g));
-  if (decode) return run_decode(p, x, M, out, out_fp32, targets, ce, amax_idx, amax_val, s);
-  return run_prefill(p, x, M, out, out_fp32, targets, ce, amax_idx, amax_val, s);
+  if (decode) return run_decode(p, x, M, out, out_fp32, targets, ce, amax_idx, amax_val, row0, parts3, s);
+  return run_prefill(p, x, M, out, out_fp32, targets, ce, amax_idx, amax_val, row0, parts3, s);
 }
 
 }  // namespace
@@ -289,6 +257,50 @@ archead_status run_forward(archead_pack *p, const void *x, int64_t M, void *out,
 namespace archead {
 
 void set_last_error_message(const char *msg) { g_last_error = msg ? msg : ""; }
+
+PrepassParams prepass_params(const archead_pack *p, const void *x, int64_t M) {
+  PrepassParams pp{};
+  pp.x = static_cast<const uint16_t *>(x);
+  pp.q_v = p->q_v;
+  pp.q_b = p->q_b;
+  pp.s_b = p->s_b;
+  pp.s_u = p->s_u;
+  pp.s_v = p->s_v;
+  pp.M = (int)M;
+  pp.d = p->d;
+  pp.g = p->g;
+  pp.rc = p->rc;
+  pp.rr = p->rr;
+  pp.rcp = p->rcp;
+  pp.rrp = p->rrp;
+  pp.lr = p->lr;
+  return pp;
+}
+
+DecodeParams decode_params(const archead_pack *p, const void *x, int64_t M_total) {
+  DecodeParams dp{};
+  dp.codes = p->codes;
+  dp.scales = p->scales;
+  dp.scodes = p->scodes;
+  dp.s_row = p->s_row;
+  dp.sc4 = p->sc4;
+  dp.G_pad2 = p->G_pad2;
+  dp.lr_codes = p->lr_codes;
+  dp.s_a = p->s_a;
+  dp.x = static_cast<const uint16_t *>(x);
+  dp.V = p->V;
+  dp.num_tiles = p->num_tiles;
+  dp.d = p->d;
+  dp.d_pad = p->d_pad;
+  dp.G_pad = p->G_pad;
+  dp.g = p->g;
+  dp.nls = p->nls;
+  dp.nls_core = p->nls_core;
+  dp.M_total = (int)M_total;
+  dp.err = p->err;
+  dp.wait_budget = p->wait_budget;
+  return dp;
+}
 
 cudaError_t opt_in_smem(const void *func, int bytes) {
   int dev = 0;
@@ -493,6 +505,39 @@ archead_status archead_forward_argmax_path(archead_pack *pack, const void *x, in
 archead_status archead_forward_argmax(archead_pack *pack, const void *x, int64_t M, int32_t *index, float *value,
                                       void *stream) {
   return archead_forward_argmax_path(pack, x, M, index, value, ARCHEAD_PATH_AUTO, stream);
+}
+
+archead_status archead_forward_lse_partial(archead_pack *pack, const void *x, int64_t M, const int32_t *targets,
+                                          int64_t row0, float *parts, archead_path path, void *stream) {
+  archead_status st = check_forward_args(pack, x, M, parts);
+  if (st != ARCHEAD_OK || M == 0) return st;
+  if (!targets || !aligned16(targets)) return ARCHEAD_ERR_INVALID_ARG;
+  if (row0 < 0 || row0 + pack->V > ((int64_t)1 << 31) - 1) return ARCHEAD_ERR_INVALID_ARG;
+  return run_forward(pack, x, M, nullptr, 0, targets, nullptr, path, static_cast<cudaStream_t>(stream), nullptr,
+                     nullptr, (int)row0, parts);
+}
+
+archead_status archead_lse_combine(const float *parts, int num_shards, int64_t M, float *ce, void *stream) {
+  if (M < 0 || num_shards < 1) return ARCHEAD_ERR_INVALID_ARG;
+  if (M == 0) return ARCHEAD_OK;
+  if (!parts || !ce || !aligned16(parts) || !aligned16(ce)) return ARCHEAD_ERR_INVALID_ARG;
+  if (M > (int64_t)1 << 30) return ARCHEAD_ERR_UNSUPPORTED;
+  AH_CUDA(launch_lse_combine(parts, num_shards, (int)M, ce, static_cast<cudaStream_t>(stream)));
+  return ARCHEAD_OK;
+}
+
+archead_status archead_argmax_combine(const float *values, const int32_t *indices, const int32_t *row0,
+                                      int num_shards, int64_t M, int32_t *index, float *value, void *stream) {
+  if (M < 0 || num_shards < 1) return ARCHEAD_ERR_INVALID_ARG;
+  if (M == 0) return ARCHEAD_OK;
+  if (!values || !indices || !row0 || !index) return ARCHEAD_ERR_INVALID_ARG;
+  if (!aligned16(values) || !aligned16(indices) || !aligned16(row0) || !aligned16(index) ||
+      (value && !aligned16(value)))
+    return ARCHEAD_ERR_INVALID_ARG;
+  if (M > (int64_t)1 << 30) return ARCHEAD_ERR_UNSUPPORTED;
+  AH_CUDA(launch_argmax_combine(values, indices, row0, num_shards, (int)M, index, value,
+                                static_cast<cudaStream_t>(stream)));
+  return ARCHEAD_OK;
 }
 
 archead_status archead_forward_host(archead_pack *pack, const void *x_host, int64_t M, void *logits_host,

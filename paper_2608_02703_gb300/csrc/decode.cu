@@ -8,15 +8,18 @@ int decode_num_units(const archead_pack *p) { return (p->num_tiles + kDecTiles -
 
 int decode_parts_per_unit() { return kDecWarps; }
 
-bool decode_supported(int d_pad, int nls, int g) { return decode_plan(d_pad, nls, g, kDecodeMaxTokens, 2).stages >= 2; }
+bool decode_supported(int d_pad, int nls, int g) {
+  return decode_plan(d_pad, nls, g, kDecodeMaxTokens, kDecStreamed2).stages >= 2;
+}
 
-// One n-tile (x resident in shared memory as fp16) while that leaves a ring
-// of at least 96 KB; otherwise the two-tile instance, which streams x through
-// the ring (very wide heads: 8 tokens of d = 16384 would take 256 KB).
-int decode_nt(int d_pad, int nls, int g, int M) {
-  if (M > 8) return 2;
-  const DecodePlan pl = decode_plan(d_pad, nls, g, M, 1);
-  return pl.stages >= 2 && pl.xs_off >= (size_t)96 * 1024 ? 1 : 2;
+// Up to 8 tokens: x resident in shared memory (fp16) while that leaves a ring
+// of at least 96 KB; otherwise, and for 9..16 tokens, the instance that
+// streams x through the ring (very wide heads: 8 tokens of d = 16384 would
+// take 256 KB).
+int decode_variant(int d_pad, int nls, int g, int M) {
+  if (M > 8) return kDecStreamed2;
+  const DecodePlan pl = decode_plan(d_pad, nls, g, M, kDecResident1);
+  return pl.stages >= 2 && pl.xs_off >= (size_t)96 * 1024 ? kDecResident1 : kDecStreamed2;
 }
 
 extern template cudaError_t launch_decode_fmt<true>(const DecodeParams &, int, cudaStream_t, bool);
@@ -24,6 +27,20 @@ template cudaError_t launch_decode_fmt<false>(const DecodeParams &, int, cudaStr
 
 cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool pdl) {
   return dp.sc4 ? launch_decode_fmt<true>(dp, grid, s, pdl) : launch_decode_fmt<false>(dp, grid, s, pdl);
+}
+
+// Opt in every instance the pack can launch: the largest token count of
+// each variant needs the most shared memory.
+cudaError_t prepare_decode(const archead_pack *p) {
+  if (!decode_supported(p->d_pad, p->nls, p->g)) return cudaSuccess;
+  DecodeParams dp = decode_params(p, nullptr, kDecodeMaxTokens);
+  for (int M : {8, kDecodeMaxTokens}) {
+    dp.M = M;
+    dp.variant = decode_variant(p->d_pad, p->nls, p->g, M);
+    const cudaError_t e = launch_decode(dp, 0, nullptr, false);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 }  // namespace archead

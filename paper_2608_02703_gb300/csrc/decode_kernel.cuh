@@ -38,18 +38,30 @@ constexpr int kDecTiles = 4;                      // 128-row tiles per unit
 constexpr int kDecMT = 4;                         // m-tiles per consumer warp (2 warps per tile)
 constexpr int kSmemLimit = 227 * 1024;
 
-// 64-wide chunks of d per ring stage, by number of 8-token n-tiles.  The
-// shared-memory plan and the kernel instance launched both take it from here.
-__host__ __device__ constexpr int stage_chunks(int NT) { return 2; }
+// Kernel instances ("variants"), chosen per launch from the token count and
+// the head's width:
+//  - kDecResident1: up to 8 tokens (one 8-token n-tile), hidden states staged
+//    once in shared memory as fp16;
+//  - kDecStreamed2: 9..16 tokens (two n-tiles), and up to 8 tokens of heads
+//    so wide that x of 8 tokens does not fit next to a working ring.  The
+//    hidden states are not kept in shared memory (16 rows of d would take
+//    most of it, leaving too shallow a ring to stream at full bandwidth):
+//    each residual stage also carries the matching 64-wide chunks of x for
+//    16 tokens, loaded by a 2-D TMA copy, and the operands stay bf16 (no fp16
+//    staging).  Its warps read codes and x from the stage as they compute and
+//    release it afterwards (the registers to copy a stage out first are not
+//    there with two n-tiles).
+// Measured alternatives that were slower on the Qwen3-8B-shaped head (and not
+// kept): 16 tokens of x resident as fp16 with a 2-chunk ring (98.4 us at
+// M = 16 against 94.8) or a 1-chunk ring with the next stage prefetched into
+// registers (114 us); 1-chunk stages for M <= 8 (98 us at M = 1 against 65).
+enum DecodeVariant { kDecResident1 = 0, kDecStreamed2 = 1 };
 
-// Instances with two n-tiles (9..16 tokens) do not keep the hidden states in
-// shared memory (16 rows of d would take most of it, leaving too shallow a
-// ring to stream at full bandwidth).  Each residual stage instead carries the
-// matching 64-wide chunks of x for 16 tokens, loaded by a 2-D TMA copy, and
-// those instances multiply bf16 operands (no fp16 staging).  Their warps read
-// codes and x from the stage as they compute and release it afterwards (the
-// registers to copy a stage out first are not there with two n-tiles).
-__host__ __device__ constexpr bool streams_x(int NT) { return NT == 2; }
+__host__ __device__ constexpr int variant_nt(int v) { return v == kDecResident1 ? 1 : 2; }
+__host__ __device__ constexpr bool streams_x(int v) { return v == kDecStreamed2; }
+// 64-wide chunks of d per ring stage.  The shared-memory plan and the kernel
+// instance launched both take it from here.
+__host__ __device__ constexpr int stage_chunks(int v) { return 2; }
 constexpr int kXChunkBytes = 16 * kChunkK * 2;  // 16 tokens x 64 of d, bf16, 128-byte swizzle
 
 // Stage geometry for SC chunks (64 of d each) per stage.
@@ -73,10 +85,10 @@ __host__ __device__ __forceinline__ int xs_row_elems(int d_pad) { return d_pad +
 // fragments, the per-group sums of x, and the barriers.  The total leaves
 // room for one pre-pass block on the same SM (programmatic dependent launch
 // overlaps the two grids) whenever the stage ring still holds 96 KB.
-static DecodePlan decode_plan(int d_pad, int nls, int g, int M, int nt) {
+static DecodePlan decode_plan(int d_pad, int nls, int g, int M, int variant) {
   DecodePlan pl{};
-  const bool xs = streams_x(nt);
-  pl.sc = stage_chunks(nt);
+  const bool xs = streams_x(variant);
+  pl.sc = stage_chunks(variant);
   const size_t stage_bytes = pl.sc == 2 ? (xs ? StageGeom<2, true>::kBytes : StageGeom<2, false>::kBytes)
                                         : (xs ? StageGeom<1, true>::kBytes : StageGeom<1, false>::kBytes);
   const size_t xs_bytes = xs ? 0 : (size_t)M * xs_row_elems(d_pad) * 2;
@@ -97,22 +109,6 @@ static DecodePlan decode_plan(int d_pad, int nls, int g, int M, int nt) {
   pl.bar_off = pl.xsum_off + xsum_bytes;
   pl.total = pl.bar_off + 256;
   return pl;
-}
-
-// Residual group promotion with the operand bias removed:
-// acc += s_row * (part + nb_tok), nb = -(operand bias) * sum of x over the
-// group, separately for rows gq (bias 1032) and gq + 8 (bias 1152; s_hi
-// carries the 1/16 of those rows' operands).
-template <int NT>
-__device__ __forceinline__ void promote_res(float (&acc)[NT][4], const float (&part)[NT][4], float s_lo, float s_hi,
-                                            const float2 (&nb_lo)[NT], const float2 (&nb_hi)[NT]) {
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt) {
-    acc[nt][0] = fmaf(s_lo, part[nt][0] + nb_lo[nt].x, acc[nt][0]);
-    acc[nt][1] = fmaf(s_lo, part[nt][1] + nb_lo[nt].y, acc[nt][1]);
-    acc[nt][2] = fmaf(s_hi, part[nt][2] + nb_hi[nt].x, acc[nt][2]);
-    acc[nt][3] = fmaf(s_hi, part[nt][3] + nb_hi[nt].y, acc[nt][3]);
-  }
 }
 
 // acc += f_lo * part (rows gq) and f_hi * part (rows gq + 8).
@@ -139,11 +135,13 @@ __device__ __forceinline__ float scale_mult_16th(uint32_t b, int sh) {
   return __uint_as_float(0x49000000u | ((b >> sh) & 15u)) - 524287.9375f;
 }
 
-// NT: n-tiles of 8 tokens; SC: 64-wide chunks per stage; GS: 16-wide k steps per group.
-template <int NT, int SC, int GS, bool kSC4>
+// VAR: DecodeVariant (n-tiles of 8 tokens, resident or streamed x); SC:
+// 64-wide chunks per stage; GS: 16-wide k steps per group.
+template <int VAR, int SC, int GS, bool kSC4>
 __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_constant__ DecodeParams p, int stages,
                                                                 int xs_off, int ts_off, int xsum_off, int bar_off) {
-  constexpr bool kStreamX = streams_x(NT);
+  constexpr int NT = variant_nt(VAR);
+  constexpr bool kStreamX = streams_x(VAR);
   constexpr bool kF16 = !kStreamX;  // fp16 operands with x staged in shared memory
   using Geom = StageGeom<SC, kStreamX>;
   constexpr int SS = 4 * SC;  // 16-wide k steps per stage
@@ -461,6 +459,22 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
               b[nt][1] = *reinterpret_cast<const uint32_t *>(q + 8);
             }
           }
+          // First k step of a group (compile-time when groups fit in a stage).
+          // Its MMAs start from the group's bias term instead of zero:
+          // nb = -(operand bias) * sum of x over the group, per token, for
+          // rows gq (bias 1032, or 136 for bf16) and gq + 8 (1152 or 136), so
+          // that the finished part is the exact-code dot product.
+          const bool first = GS <= SS ? (ks % GS == 0) : (ks == 0 && (s % (GS / SS)) == 0);
+          float2 nb_lo[NT], nb_hi[NT];
+          if (first) {
+            const int ggl = GS <= SS ? s * (SS / GS) + ks / GS : s / (GS / SS);  // group index along d
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+              const int o = ggl * kDecodeMaxTokens + 8 * nt + 2 * cq;
+              nb_lo[nt] = *reinterpret_cast<const float2 *>(xsum_s + o);
+              nb_hi[nt] = *reinterpret_cast<const float2 *>(xsum_s + ng * kDecodeMaxTokens + o);
+            }
+          }
 #pragma unroll
           for (int mt = 0; mt < kDecMT; ++mt) {
             const uint4 wv = w[kStreamX ? 0 : c][mt];
@@ -470,18 +484,16 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
               unpack_int4x8_f16(word, a);
             else
               unpack_int4x8_biased(word, a);
-            // First k step of a group: compile-time when groups fit in a stage.
-            const bool first = GS <= SS ? (ks % GS == 0) : (ks == 0 && (s % (GS / SS)) == 0);
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
               if (kF16) {
                 if (first)
-                  mma_f16_16816_zero(part[mt][nt], a, b[nt][0], b[nt][1]);
+                  mma_f16_16816_c(part[mt][nt], a, b[nt][0], b[nt][1], nb_lo[nt], nb_hi[nt]);
                 else
                   mma_f16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
               } else {
                 if (first)
-                  mma_bf16_16816_zero(part[mt][nt], a, b[nt][0], b[nt][1]);
+                  mma_bf16_16816_c(part[mt][nt], a, b[nt][0], b[nt][1], nb_lo[nt], nb_hi[nt]);
                 else
                   mma_bf16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
               }
@@ -491,18 +503,9 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
           // GS/SS stages otherwise.
           const bool boundary = GS <= SS ? ((ks + 1) % GS == 0) : (ks == SS - 1 && ((s + 1) % (GS / SS)) == 0);
           if (boundary) {
-            const int gi = GS <= SS ? ks / GS : 0;                               // group within the stage
-            const int ggl = GS <= SS ? s * (SS / GS) + ks / GS : s / (GS / SS);  // group index along d
-            float2 nb_lo[NT], nb_hi[NT];
+            const int gi = GS <= SS ? ks / GS : 0;  // group within the stage
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-              const int o = ggl * kDecodeMaxTokens + 8 * nt + 2 * cq;
-              nb_lo[nt] = *reinterpret_cast<const float2 *>(xsum_s + o);
-              nb_hi[nt] = *reinterpret_cast<const float2 *>(xsum_s + ng * kDecodeMaxTokens + o);
-            }
-#pragma unroll
-            for (int mt = 0; mt < kDecMT; ++mt)
-              promote_res<NT>(acc[mt], part[mt], s_lo[gi][mt], s_hi[gi][mt], nb_lo, nb_hi);
+            for (int mt = 0; mt < kDecMT; ++mt) promote<NT>(acc[mt], part[mt], s_lo[gi][mt], s_hi[gi][mt]);
           }
         }
       }
@@ -692,7 +695,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
 #pragma unroll
         for (int tl = 0; tl < 2; ++tl) {
           const int tok = nt * 8 + 2 * cq + tl;
-          const int tgt = tok < p.M ? p.targets[p.m0 + tok] : -1;
+          const int tgt = tok < p.M ? p.targets[p.m0 + tok] - p.row0 : -1;  // this pack's row numbering
           float vals[2 * kDecMT];
           float mx = -INFINITY;
 #pragma unroll
@@ -722,11 +725,11 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
   }
 }
 
-template <int NT, int SC, int GS, bool kSC4>
+template <int VAR, int SC, int GS, bool kSC4>
 static cudaError_t launch_t(const DecodeParams &dp, int grid, cudaStream_t s, const DecodePlan &pl, bool pdl) {
-  auto kern = decode_kernel<NT, SC, GS, kSC4>;
+  auto kern = decode_kernel<VAR, SC, GS, kSC4>;
   cudaError_t e = opt_in_smem(reinterpret_cast<const void *>(kern), (int)pl.total);
-  if (e != cudaSuccess) return e;
+  if (e != cudaSuccess || grid == 0) return e;  // grid 0: opt-in only (prepare_decode)
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kDecThreads);
@@ -741,31 +744,31 @@ static cudaError_t launch_t(const DecodeParams &dp, int grid, cudaStream_t s, co
                             (int)pl.bar_off);
 }
 
-template <int NT, int SC, bool kSC4>
+template <int VAR, bool kSC4>
 static cudaError_t launch_g(const DecodeParams &dp, int grid, cudaStream_t s, const DecodePlan &pl, bool pdl) {
+  constexpr int SC = stage_chunks(VAR);
   switch (dp.g) {
-    case 32: return launch_t<NT, SC, 2, kSC4>(dp, grid, s, pl, pdl);
-    case 64: return launch_t<NT, SC, 4, kSC4>(dp, grid, s, pl, pdl);
-    case 128: return launch_t<NT, SC, 8, kSC4>(dp, grid, s, pl, pdl);
-    case 256: return launch_t<NT, SC, 16, kSC4>(dp, grid, s, pl, pdl);
+    case 32: return launch_t<VAR, SC, 2, kSC4>(dp, grid, s, pl, pdl);
+    case 64: return launch_t<VAR, SC, 4, kSC4>(dp, grid, s, pl, pdl);
+    case 128: return launch_t<VAR, SC, 8, kSC4>(dp, grid, s, pl, pdl);
+    case 256: return launch_t<VAR, SC, 16, kSC4>(dp, grid, s, pl, pdl);
   }
   return cudaErrorInvalidValue;
 }
 
 // One packed format's kernel instances (INT8 in decode.cu, SC4 in decode_sc4.cu,
-// so that the two sets compile in parallel).
+// so that the two sets compile in parallel).  grid == 0 only opts the
+// instance into its shared memory (no launch).
 template <bool kSC4>
 cudaError_t launch_decode_fmt(const DecodeParams &dp, int grid, cudaStream_t s, bool pdl) {
-  const DecodePlan pl = decode_plan(dp.d_pad, dp.nls, dp.g, dp.M, dp.NT);
-  if (pl.stages < 2) return cudaErrorInvalidValue;
-  static_assert(stage_chunks(1) >= 1 && stage_chunks(2) >= 1, "stage width");
-  if ((dp.NT != 1 && dp.NT != 2) || (dp.NT == 1 && dp.M > 8) || pl.sc != stage_chunks(dp.NT))
-    return cudaErrorInvalidValue;
-  if (dp.NT == 1) return launch_g<1, stage_chunks(1), kSC4>(dp, grid, s, pl, pdl);
-  static_assert(streams_x(2) && !streams_x(1), "two n-tiles stream x");
+  const DecodePlan pl = decode_plan(dp.d_pad, dp.nls, dp.g, dp.M, dp.variant);
+  if (pl.stages < 2 || pl.sc != stage_chunks(dp.variant)) return cudaErrorInvalidValue;
+  if (dp.M < 1 || dp.M > (variant_nt(dp.variant) == 1 ? 8 : 16)) return cudaErrorInvalidValue;
+  if (dp.variant == kDecResident1) return launch_g<kDecResident1, kSC4>(dp, grid, s, pl, pdl);
+  if (dp.variant != kDecStreamed2) return cudaErrorInvalidValue;
   DecodeParams dx = dp;
-  if (!make_tma_map_bf16(&dx.tmap_x, dp.x, dp.M_total, dp.d, 16)) return cudaErrorInvalidValue;
-  return launch_g<2, stage_chunks(2), kSC4>(dx, grid, s, pl, pdl);
+  if (grid > 0 && !make_tma_map_bf16(&dx.tmap_x, dp.x, dp.M_total, dp.d, 16)) return cudaErrorInvalidValue;
+  return launch_g<kDecStreamed2, kSC4>(dx, grid, s, pl, pdl);
 }
 
 

@@ -36,8 +36,8 @@ __device__ __forceinline__ uint32_t lop3_and_or(uint32_t a, uint32_t b, uint32_t
 }
 
 // Biased operands: each half is 136 + code (128..143, exact in bf16).  The
-// decode kernel multiplies these directly and removes 136 * sum(x) per group
-// in fp32 at promotion time.
+// decode kernel multiplies these directly; the MMAs of each quantisation
+// group start from -136 * sum(x) over the group, which removes the bias.
 __device__ __forceinline__ void unpack_int4x8_biased(uint32_t w, uint32_t (&a)[4]) {
   const uint32_t kMask = 0x000F000Fu;
   const uint32_t kMagic = 0x43004300u;  // bf16 128.0 | 128.0
@@ -54,8 +54,8 @@ constexpr float kInt4Bias = 136.0f;
 // so a word's eight nibbles need one shift and four LOP3s.  Registers a[0],
 // a[2] (rows gq of the m16n8k16 A fragment) hold 1024 + n = 1032 + code;
 // a[1], a[3] (rows gq + 8) hold 1024 + 16 n = 1152 + 16 code.  The kernel
-// removes 1032 * sum(x) resp. 1152 * sum(x) per group and scales rows gq + 8
-// by 1/16 at promotion.
+// starts each group's MMAs from -1032 * sum(x) resp. -1152 * sum(x) and
+// scales rows gq + 8 by 1/16 at promotion.
 constexpr float kF16BiasLo = 1032.0f;
 constexpr float kF16BiasHi = 1152.0f;
 
@@ -125,6 +125,18 @@ __device__ __forceinline__ void mma_bf16_16816_zero(float (&d)[4], const uint32_
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(0.f));
 }
 
+// Same with the accumulator input taken from (c_lo.x, c_lo.y, c_hi.x, c_hi.y)
+// (the first k step of a group, started from the group's bias term).
+__device__ __forceinline__ void mma_bf16_16816_c(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1,
+                                                 float2 c_lo, float2 c_hi) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%11,%12,%13};\n"
+      : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(c_lo.x), "f"(c_lo.y), "f"(c_hi.x),
+        "f"(c_hi.y));
+}
+
 // fp16 x fp16 -> fp32 variants (the decode kernel's residual operands).
 __device__ __forceinline__ void mma_f16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
   asm volatile(
@@ -140,6 +152,16 @@ __device__ __forceinline__ void mma_f16_16816_zero(float (&d)[4], const uint32_t
       "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%10,%10,%10};\n"
       : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(0.f));
+}
+
+__device__ __forceinline__ void mma_f16_16816_c(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1,
+                                                float2 c_lo, float2 c_hi) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%11,%12,%13};\n"
+      : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(c_lo.x), "f"(c_lo.y), "f"(c_hi.x),
+        "f"(c_hi.y));
 }
 
 // ---------------------------------------------------------------------------

@@ -68,12 +68,13 @@ struct DecodeParams {
   int sc4, G_pad2;      // SC4 format flag; byte rows of scale codes per tile
   int M;                // tokens in this chunk (1..16)
   int m0;               // index of the chunk's first token
-  int NT;               // n-tiles of 8 tokens (1 or 2)
+  int variant;          // kernel instance (decode_variant)
   void *out;            // logits [M_total][V] (NULL in CE mode)
   int out_fp32;
   // CE mode (out == NULL, argmax == 0) or greedy mode (out == NULL, argmax != 0)
   int argmax;
-  const int32_t *targets;  // [M_total]
+  const int32_t *targets;  // [M_total], global vocabulary rows
+  int row0;                // global row of this pack's first row (vocabulary shards; 0 otherwise)
   float2 *ce_part;         // [num_units][M_total] (max, sum exp)
   float *ce_tlogit;        // [M_total]
   int M_total;
@@ -139,6 +140,11 @@ struct archead_pack {
 
 namespace archead {
 
+// Kernel parameters filled from the pack (the call-specific fields -- outputs,
+// token chunk, workspace pointers -- are left for the caller).
+PrepassParams prepass_params(const archead_pack *p, const void *x, int64_t M);
+DecodeParams decode_params(const archead_pack *p, const void *x, int64_t M_total);
+
 // Kernel launchers (each returns the launch's cudaError_t).
 // res_scales and core_u are the canonical arrays of the pack's format (SC4:
 // 4-bit scale codes and 5-bit core codes; row_scale its residual row scales).
@@ -156,6 +162,9 @@ size_t prepass_smem(int M);  // dynamic shared memory of one pre-pass block
 size_t prepass_partial_bytes(int M, int lr, int d);
 // pdl: launch as a programmatic dependent of the immediately preceding pre-pass grid.
 cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool pdl);
+// Shared-memory opt-in (and so module loading) of every decode kernel
+// instance this pack can launch for 1..16 tokens, done ahead of any launch.
+cudaError_t prepare_decode(const archead_pack *p);
 // Tensor map of a bf16 [rows][cols] row-major matrix: box 64 columns x
 // box_rows rows, 128-byte swizzle, zero fill out of bounds.  False if the
 // driver entry point is missing or the encoder rejects the layout (base or
@@ -164,9 +173,12 @@ bool make_tma_map_bf16(CUtensorMap *map, const void *base, int64_t rows, int64_t
 int decode_num_units(const archead_pack *p);
 int decode_parts_per_unit();
 bool decode_supported(int d_pad, int nls, int g);
-int decode_nt(int d_pad, int nls, int g, int M);  // n-tiles of 8 tokens of the instance to launch for M tokens
+// Kernel instance to launch for M <= 16 tokens (0: one 8-token tile, x
+// resident; 1: two tiles, x resident; 2: two tiles, x streamed).
+int decode_variant(int d_pad, int nls, int g, int M);
 cudaError_t launch_prefill(const archead_pack *pk, const void *x, int M, const uint16_t *T, void *out, int out_fp32,
-                           bool argmax, const int32_t *targets, float2 *ce_part, float *ce_tlogit, cudaStream_t s);
+                           bool argmax, const int32_t *targets, int row0, float2 *ce_part, float *ce_tlogit,
+                           cudaStream_t s);
 int prefill_parts_per_vt();
 // Greedy second pass: per token the largest (value, row) over the partials,
 // lowest row on ties.
@@ -174,6 +186,14 @@ cudaError_t launch_argmax_finalize(const float2 *part, int num_parts, int M, int
                                    cudaStream_t s);
 cudaError_t launch_ce_finalize(const float2 *part, int num_parts, const float *tlogit, const int32_t *targets,
                                int64_t V, int M, float *ce, int *err, cudaStream_t s);
+// Vocabulary shards: per token (max, sum of exp(y - max), target logit or
+// -inf when the target is not one of this shard's rows [row0, row0 + V)).
+cudaError_t launch_lse_partial_finalize(const float2 *part, int num_parts, const float *tlogit,
+                                        const int32_t *targets, int64_t row0, int64_t V, int M, float *parts3,
+                                        cudaStream_t s);
+cudaError_t launch_lse_combine(const float *parts3, int num_shards, int M, float *ce, cudaStream_t s);
+cudaError_t launch_argmax_combine(const float *values, const int32_t *indices, const int32_t *row0, int num_shards,
+                                  int M, int32_t *index, float *value, cudaStream_t s);
 cudaError_t launch_wait_timeout_probe(int *err, int64_t budget, cudaStream_t s);
 
 // Opt `func` into `bytes` of dynamic shared memory on the current device:

@@ -37,6 +37,9 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratch
 // device current.  In host code the symbol is only a host-side stand-in: a
 // kernel handed &g_noalloc_scratch would fault (or silently touch host memory
 // where the device can reach it), so kernels only ever get this address.
+// The address is cached for the life of the process: calls after a
+// cudaDeviceReset of that device are not supported (its module, and so the
+// array, may be loaded elsewhere afterwards).
 static void *g_scratch_dev[kNoallocMaxDevices];
 static std::mutex g_scratch_mu;
 
@@ -98,55 +101,25 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
 
   // The counters are the only state that must start at zero.
   e = cudaMemsetAsync(counters, 0, (size_t)pairs * sizeof(int), s);
+  // Every decode instance this pack can use (one or two 8-token tiles) is
+  // opted into its shared memory here, so that a first call at any M leaves
+  // nothing for a later call at another M to set up (inside a capture, say).
+  if (e == cudaSuccess) e = prepare_decode(pack);
 
-  PrepassParams pp{};
-  pp.x = static_cast<const uint16_t *>(x);
-  pp.q_v = pack->q_v;
-  pp.q_b = pack->q_b;
-  pp.s_b = pack->s_b;
-  pp.s_u = pack->s_u;
-  pp.s_v = pack->s_v;
-  pp.M = (int)M;
-  pp.d = pack->d;
-  pp.g = pack->g;
-  pp.rc = pack->rc;
-  pp.rr = pack->rr;
-  pp.rcp = pack->rcp;
-  pp.rrp = pack->rrp;
-  pp.lr = pack->lr;
+  PrepassParams pp = prepass_params(pack, x, M);
   pp.partial = partial;
   pp.counters = counters;
   pp.ts = ts;
   pp.T = nullptr;
   if (e == cudaSuccess) e = launch_prepass(pp, s, nullptr);  // no profiling events on this path
 
-  DecodeParams dp{};
-  dp.codes = pack->codes;
-  dp.scales = pack->scales;
-  dp.scodes = pack->scodes;
-  dp.s_row = pack->s_row;
-  dp.sc4 = pack->sc4;
-  dp.G_pad2 = pack->G_pad2;
-  dp.lr_codes = pack->lr_codes;
-  dp.s_a = pack->s_a;
-  dp.x = static_cast<const uint16_t *>(x);
+  DecodeParams dp = decode_params(pack, x, M);
   dp.ts = ts;
-  dp.V = pack->V;
-  dp.num_tiles = pack->num_tiles;
-  dp.d = pack->d;
-  dp.d_pad = pack->d_pad;
-  dp.G_pad = pack->G_pad;
-  dp.g = pack->g;
-  dp.nls = pack->nls;
-  dp.nls_core = pack->nls_core;
   dp.M = (int)M;
   dp.m0 = 0;
-  dp.NT = decode_nt(pack->d_pad, pack->nls, pack->g, (int)M);
+  dp.variant = decode_variant(pack->d_pad, pack->nls, pack->g, (int)M);
   dp.out = logits;
   dp.out_fp32 = out_dtype == ARCHEAD_OUT_FP32;
-  dp.M_total = (int)M;
-  dp.err = pack->err;
-  dp.wait_budget = pack->wait_budget;
   const int units = decode_num_units(pack);
   if (e == cudaSuccess) e = launch_decode(dp, units < pack->sm_count ? units : pack->sm_count, s, pack->lr > 0);
   if (e != cudaSuccess) {

@@ -56,7 +56,8 @@ struct PrefillParams {
   int sc4, G_pad2;
   void *out;
   int out_fp32;
-  const int32_t *targets;
+  const int32_t *targets;  // global vocabulary rows
+  int row0;                // global row of this pack's first row (vocabulary shards; 0 otherwise)
   float2 *ce_part;   // [num_vt * 4][M]
   float *ce_tlogit;  // [M]
   int *err;
@@ -497,7 +498,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           const int m = m0 + 4 * lane + j;
-          tg[j] = m < p.M ? p.targets[m] : -1;
+          tg[j] = m < p.M ? p.targets[m] - p.row0 : -1;  // this pack's row numbering
           hit |= tg[j] >= rowbase && tg[j] < rowbase + 32;
         }
         if (__any_sync(0xffffffffu, hit)) {
@@ -567,8 +568,8 @@ done:
 // One packed format's kernel instances (INT8 in prefill.cu, SC4 in prefill_sc4.cu).
 template <bool kSC4>
 cudaError_t launch_prefill_fmt(const archead_pack *pk, const void *x, int M, const uint16_t *T, void *out,
-                               int out_fp32, bool argmax, const int32_t *targets, float2 *ce_part, float *ce_tlogit,
-                               cudaStream_t s) {
+                               int out_fp32, bool argmax, const int32_t *targets, int row0, float2 *ce_part,
+                               float *ce_tlogit, cudaStream_t s) {
   PrefillParams p{};
   if (!make_tma_map_bf16(&p.tmap_x, x, M, pk->d, 128)) return cudaErrorInvalidValue;
   const int kt = 2 * (pk->rcp + pk->rrp);
@@ -597,6 +598,7 @@ cudaError_t launch_prefill_fmt(const archead_pack *pk, const void *x, int M, con
   p.out = out;
   p.out_fp32 = out_fp32;
   p.targets = targets;
+  p.row0 = row0;
   p.ce_part = ce_part;
   p.ce_tlogit = ce_tlogit;
   p.err = pk->err;

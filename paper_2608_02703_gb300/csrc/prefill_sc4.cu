@@ -5,6 +5,6 @@
 namespace archead {
 
 template cudaError_t launch_prefill_fmt<true>(const archead_pack *, const void *, int, const uint16_t *, void *, int,
-                                              bool, const int32_t *, float2 *, float *, cudaStream_t);
+                                              bool, const int32_t *, int, float2 *, float *, cudaStream_t);
 
 }  // namespace archead
