@@ -9,8 +9,9 @@ default workload is the Qwen3-8B-shaped head (V=151936, d=4096, r_c=128,
 r_r=32, g=128) at M=1 token (decode); the same line also carries the decode
 sweep M=2..16, the M=4096 prefill (logits and fused cross entropy), a dense
 BF16 cuBLAS head on the same shapes, the batch sweep M=1..8192 through both
-kernels, the same head in the paper's own packed format, and the
-Gemma-4-E4B-shaped head.
+kernels, the same head in the paper's own packed format, the
+Gemma-4-E4B-shaped head, the tiny head (a latency entry beside the oracle)
+and the headline figures of those blocks again as flat top-level keys.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -400,9 +401,74 @@ def run_ours(args, rank, world, local_rank):
     if not args.no_extras and args.workload == "qwen3-8b-decode":
         result["sc4"] = sc4_block(peaks, world, local_rank)
         result["gemma"] = gemma_block(peaks, world, local_rank)
+        result["tiny"] = tiny_block(world, local_rank, with_oracle=rank == 0 and world == 1)
+        result.update(flat_keys(result))
     if rank == 0 and not args.no_cpu_baseline and world == 1:
         result["cpu_baseline"] = cpu_baseline(wl, x_np, M, budget_s=args.cpu_budget)
     return result
+
+
+def tiny_block(world, local_rank, with_oracle=True):
+    """The tiny head (V=4096, d=512, r_c=64, r_r=16, g=64) at M=4: a latency
+    entry next to the oracle on the same workload.  Its 1.5 MB pack stays in
+    the 129 MB L2, so no roofline fraction is claimed for it."""
+    import torch
+
+    from paper_2608_02703_gb300 import archead
+    from synth import make_hidden
+
+    wl = Workload("tiny")
+    pack = wl.open()
+    M = 4
+    x_np = make_hidden(wl.shape.d, M, seed=1, n_outliers=wl.shape.n_outliers)
+    x = torch.from_numpy(x_np.view(np.int16)).cuda()
+    y = torch.empty((M, wl.shape.V), dtype=torch.bfloat16, device="cuda")
+    fn = lambda: archead.archead_forward(pack, x, M, y, archead.OUT_BF16)  # noqa: E731
+    k = 2000
+    secs = max_over_ranks(timed_loop(fn, k, 20, world), world, torch.device("cuda", local_rank))
+    res = {"workload": "tiny head (V=4096, d=512, r_c=64, r_r=16, g=64), decode M=4, logits bf16",
+           "M": M, "us_per_call": round(secs / k * 1e6, 2), "tokens_s": round(world * M * k / secs, 1),
+           "packed_bytes": packed_bytes(wl.shape),
+           "note": "L2-resident (packed head 1.5 MB < 129 MB L2): a latency figure, no roofline claim"}
+    st = archead.archead_sync_status(pack)
+    res["status"] = archead.archead_status_string(st)
+    pack.close()
+    if with_oracle:
+        import oracle
+
+        t = min(oracle_rows_time(wl.head, wl.shape, x_np, wl.shape.V) for _ in range(3))
+        res["oracle"] = {"us_per_call": round(t * 1e6, 1), "cores": oracle.threads(),
+                         "sample": "the whole forward (all 4096 rows, M=4), best of 3"}
+    return res
+
+
+def flat_keys(result):
+    """The headline numbers of the nested blocks as top-level scalars."""
+    out = {}
+    pf = result.get("prefill") or {}
+    for mode in ("logits", "ce"):
+        if mode in pf:
+            out[f"qwen_prefill_m{pf['M']}_{mode}_ms"] = pf[mode]["ms_per_call"]
+            out[f"qwen_prefill_m{pf['M']}_{mode}_frac_bf16_peak"] = pf[mode]["frac_bf16_peak"]
+    for row in result.get("decode_sweep") or []:
+        out[f"qwen_decode_m{row['M']}_us"] = row["us_per_call"]
+        out[f"qwen_decode_m{row['M']}_kernel_frac_hbm"] = row["frac_hbm"]
+    for blk, name in (("sc4", "qwen_sc4"), ("gemma", "gemma")):
+        b = result.get(blk) or {}
+        for row in b.get("decode_sweep") or []:
+            out[f"{name}_decode_m{row['M']}_us"] = row["us_per_call"]
+            out[f"{name}_decode_m{row['M']}_kernel_frac_hbm"] = row["frac_hbm"]
+        bp = b.get("prefill") or {}
+        for mode in ("logits", "ce"):
+            if mode in bp:
+                out[f"{name}_prefill_m{bp['M']}_{mode}_ms"] = bp[mode]["ms_per_call"]
+                out[f"{name}_prefill_m{bp['M']}_{mode}_frac_bf16_peak"] = bp[mode]["frac_bf16_peak"]
+    t = result.get("tiny") or {}
+    if "us_per_call" in t:
+        out["tiny_m4_us"] = t["us_per_call"]
+        if "oracle" in t:
+            out["tiny_m4_oracle_us"] = t["oracle"]["us_per_call"]
+    return out
 
 
 def gemma_block(peaks, world, local_rank):

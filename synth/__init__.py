@@ -13,4 +13,5 @@ from .inputs import (  # noqa: F401
     make_hidden,
     make_targets,
     head_nbytes_canonical,
+    with_extreme_codes,
 )

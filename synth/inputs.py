@@ -196,6 +196,45 @@ def _make_head_sc4(shape: HeadShape, seed: int) -> Dict[str, np.ndarray]:
     return {k: np.ascontiguousarray(v) for k, v in head.items()}
 
 
+def with_extreme_codes(head: Dict[str, np.ndarray], shape: HeadShape, seed: int = 0,
+                       frac: float = 0.125) -> Dict[str, np.ndarray]:
+    """A copy of a packed head with the most negative code of each factor
+    array planted: INT8 -128 in core_v, corr_a and corr_b (and core_u in the
+    INT8 format), the 5-bit code -16 in core_u5 (the paper's format), and
+    INT4 -8 in every residual code of row 0.  A seeded fraction `frac` of the
+    entries, plus the whole first row and first column of each array, are
+    overwritten; everything else is left as drawn.  The symmetric generators
+    above draw INT8 codes in [-127, 127], so -128 only appears this way."""
+    out = {k: v.copy() for k, v in head.items()}
+    rng = _streams(seed + 3_000_017, ("mask",))["mask"]
+
+    def plant(a: np.ndarray, value) -> None:
+        if a.size == 0:
+            return
+        mask = rng.random(a.shape) < frac
+        mask[0, :] = True
+        mask[:, 0] = True
+        a[mask] = value
+
+    for name in ("core_v", "corr_a", "corr_b") + (("core_u",) if shape.fmt != "sc4" else ()):
+        plant(out[name], np.int8(-128))
+    if shape.fmt == "sc4" and shape.core_rank > 0:
+        # code j of a row lives in bits 5j..5j+4 of the row's little-endian
+        # bit string; -16 is 0b10000 in five-bit two's complement.
+        bits = np.unpackbits(out["core_u5"], axis=1, bitorder="little")
+        codes = np.zeros((shape.V, shape.core_rank), dtype=bool)
+        plant_mask = rng.random(codes.shape) < frac
+        plant_mask[0, :] = True
+        plant_mask[:, 0] = True
+        rows, cols = np.nonzero(plant_mask)
+        for b in range(4):
+            bits[rows, 5 * cols + b] = 0
+        bits[rows, 5 * cols + 4] = 1
+        out["core_u5"] = np.ascontiguousarray(np.packbits(bits, axis=1, bitorder="little")[:, :shape.core_u5_bytes])
+    out["res_codes"][0, :] = 0x88  # both nibbles -8
+    return {k: np.ascontiguousarray(v) for k, v in out.items()}
+
+
 def head_nbytes_canonical(head: Dict[str, np.ndarray]) -> int:
     """Sum of numel * element size over the canonical arrays."""
     return int(sum(a.nbytes for a in head.values()))

@@ -103,3 +103,18 @@ def check_greedy(idx: np.ndarray, val: np.ndarray, ref: np.ndarray, where: str =
     picked = ref[np.arange(M), idx]
     assert np.all(srt[:, -1] - picked <= 2 * tol), f"{where}: greedy index names a row far below the maximum"
     assert np.all(np.abs(val - picked) <= tol), f"{where}: greedy value max|d|={np.max(np.abs(val - picked)):.3e}"
+
+
+def ce_bound(ref: dict) -> np.ndarray:
+    """Per-token CE bar: CE_ABS, widened where the logits are so large that
+    fp32 cannot resolve it.  The kernels carry each logit in fp32 and build
+    it from sums whose terms reach CE_REL_LOGIT^-1 times the logit's own
+    size (biased residual operands, the bf16 hi/lo split of t), so a logit
+    of size L is resolved to about CE_REL_LOGIT * L; CE, a difference of two
+    logits, gets twice that.  At logit rms ~2 the widening is below 1e-4."""
+    big = np.maximum(np.abs(ref["target_logit"]), np.abs(ref["ce"] + ref["target_logit"]))
+    return CE_ABS + 2.0 * CE_REL_LOGIT * big
+
+
+# Relative resolution of a logit computed by the kernels (see ce_bound).
+CE_REL_LOGIT = 2.0 ** -14

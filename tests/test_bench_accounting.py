@@ -37,3 +37,22 @@ def test_traffic_is_used_only_for_the_sources_it_was_captured_with(tmp_path, mon
     assert bench.captured_traffic("decode", "qwen3-8b-decode", 16) is None      # no capture at this M
     assert bench.captured_traffic("prefill", "qwen3-8b-prefill", 1024) is None  # sources changed since
 
+
+
+def test_flat_keys_repeat_the_nested_headline_figures():
+    res = {
+        "prefill": {"M": 4096, "logits": {"ms_per_call": 4.2, "frac_bf16_peak": 0.66},
+                    "ce": {"ms_per_call": 4.8, "frac_bf16_peak": 0.58}},
+        "decode_sweep": [{"M": 1, "us_per_call": 68.5, "frac_hbm": 0.77}, {"M": 16, "us_per_call": 80.0, "frac_hbm": 0.7}],
+        "sc4": {"decode_sweep": [{"M": 1, "us_per_call": 66.0, "frac_hbm": 0.72}],
+                "prefill": {"M": 4096, "logits": {"ms_per_call": 3.9, "frac_bf16_peak": 0.69}}},
+        "gemma": {"decode_sweep": [], "prefill": {"M": 2048, "ce": {"ms_per_call": 3.0, "frac_bf16_peak": 0.51}}},
+        "tiny": {"us_per_call": 9.5, "oracle": {"us_per_call": 12000.0}},
+    }
+    flat = bench.flat_keys(res)
+    assert flat["qwen_prefill_m4096_logits_ms"] == 4.2 and flat["qwen_prefill_m4096_ce_frac_bf16_peak"] == 0.58
+    assert flat["qwen_decode_m16_us"] == 80.0 and flat["qwen_decode_m1_kernel_frac_hbm"] == 0.77
+    assert flat["qwen_sc4_decode_m1_us"] == 66.0 and flat["qwen_sc4_prefill_m4096_logits_ms"] == 3.9
+    assert flat["gemma_prefill_m2048_ce_ms"] == 3.0
+    assert flat["tiny_m4_us"] == 9.5 and flat["tiny_m4_oracle_us"] == 12000.0
+    assert all(not isinstance(v, (dict, list)) for v in flat.values())

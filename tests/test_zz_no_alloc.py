@@ -4,9 +4,10 @@ graph capture under a pool that forbids new allocations, latency-critical
 loops).  Its scratch is a fixed 512 KiB array inside the library instead of the
 pack's cudaMalloc-grown workspace.
 
-The test compares it, through the C ABI, with archead_forward on the same
-inputs, on two calls in a row (the second call finds the first call's data in
-the shared array).  This file is collected last on purpose.
+The tests call it through the C ABI and check its logits against the fp64
+oracle under the same bars as every other parity test, on two calls in a row
+(the second call finds the first call's data in the shared array; both must
+give the same bits).  This file is collected last on purpose.
 """
 
 import zlib
@@ -50,18 +51,21 @@ def _run_noalloc(pack, x_bits, out_dtype):
 
 @pytest.mark.parametrize("shape", SHAPES, ids=lambda s: f"V{s.V}_d{s.d}_g{s.group_size}_{s.fmt}")
 @pytest.mark.parametrize("out_dtype", [archead.OUT_FP32, archead.OUT_BF16])
-def test_noalloc_matches_forward_on_two_calls_in_a_row(shape, out_dtype):
+def test_noalloc_matches_oracle_on_two_calls_in_a_row(shape, out_dtype):
     head = make_head(shape, seed=zlib.crc32(repr(shape).encode()) % 1000)
     pack = archead.archead_pack_create(head, shape)
     try:
         for M, seed in ((7, 1), (16, 2), (1, 3)):
             x = make_hidden(shape.d, M, seed=seed)
-            ref = gu.forward(pack, x, out_dtype, archead.PATH_DECODE)
+            ref = oracle.logits(head, shape, x)
             first = _run_noalloc(pack, x, out_dtype)
             second = _run_noalloc(pack, x, out_dtype)
+            bf16 = out_dtype == archead.OUT_BF16
             for got in (first, second):
-                gu.check_logits(got, ref, bf16=False, where=f"noalloc M={M}")
+                gu.check_logits(got, ref, bf16=bf16, where=f"noalloc M={M}")
             assert np.array_equal(first, second)
+            # and the same bits as the allocating entry point
+            assert np.array_equal(first, gu.forward(pack, x, out_dtype, archead.PATH_DECODE))
     finally:
         pack.close()
 
@@ -128,5 +132,36 @@ def test_noalloc_forward_replays_as_a_cuda_graph():
             assert archead.archead_sync_status(pack) == archead.OK
             got = y.cpu().numpy().astype(np.float64)
             gu.check_logits(got, oracle.logits(head, shape, x), where=f"graph replay seed={seed}")
+    finally:
+        pack.close()
+
+
+def test_noalloc_capture_after_warm_up_at_another_token_count():
+    """A warm-up call at M = 1 prepares every decode instance the pack can
+    use (one and two 8-token tiles), so a capture at M = 16 does no first-time
+    set-up inside the capture; the replay is checked against the oracle."""
+    import torch
+
+    shape = SHAPES[3]
+    head = make_head(shape, seed=17)
+    pack = archead.archead_pack_create(head, shape)
+    try:
+        x1 = gu.to_dev(make_hidden(shape.d, 1, seed=17))
+        y1 = torch.zeros((1, shape.V), dtype=torch.float32, device="cuda")
+        archead.archead_forward_decode_noalloc(pack, x1, 1, y1, archead.OUT_FP32)
+        torch.cuda.synchronize()
+        M = 16
+        xd = torch.zeros((M, shape.d), dtype=torch.int16, device="cuda")
+        y = torch.zeros((M, shape.V), dtype=torch.bfloat16, device="cuda")
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            archead.archead_forward_decode_noalloc(pack, xd, M, y, archead.OUT_BF16)
+        x = make_hidden(shape.d, M, seed=18)
+        xd.copy_(torch.from_numpy(x.view(np.int16)))
+        g.replay()
+        torch.cuda.synchronize()
+        assert archead.archead_sync_status(pack) == archead.OK
+        gu.check_logits(y.float().cpu().numpy().astype(np.float64), oracle.logits(head, shape, x), bf16=True,
+                        where="capture at M=16 after warm-up at M=1")
     finally:
         pack.close()
