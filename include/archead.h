@@ -315,6 +315,53 @@ ARCHEAD_API archead_status archead_debug_wait_timeout(archead_pack *pack, void *
 ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pack *pack, const void *x, int64_t M,
                                                           void *logits, archead_out_dtype out_dtype, void *stream);
 
+/*
+ * Offline construction of a packed head (paper, Section 3.4, Algorithm 1;
+ * Appendix B steps 3-7): the quantisation and packing steps, on the device.
+ * The dense linear algebra around them (H^T H, the eigendecomposition of the
+ * damped covariance, the randomized SVDs of W and of E T_p) is done by library
+ * routines in paper_2608_02703_gb300/construct.py, which calls these.  All
+ * pointers are device memory; inputs are fp32, row-major.
+ *
+ * archead_quantize_symmetric: codes int8 [rows][cols] and fp16 scales
+ *   [rows/group_rows][cols/group_cols] of x, one scale per group_rows x
+ *   group_cols block: scale = fp16(max|x| / qmax) (fp32 division, round to
+ *   nearest even), code = clamp(rint(x / scale), -qmax, qmax) with the
+ *   division in fp32 and ties to even; code 0 where the scale is 0.
+ *   bits 8 (qmax 127: Q_8 and the INT8 correction factors), 5 (qmax 15: the
+ *   paper's Q_5 core left factor) or 4 (qmax 7: the INT4 residual).
+ *   Row-wise: group_rows = 1, group_cols = cols; per column: group_rows =
+ *   rows, group_cols = 1; B_w^T group-wise along d: group_rows = g,
+ *   group_cols = 1; residual with one scale per group: 1 x g.
+ * archead_quantize_residual_sc4: the residual in the paper's format: per row
+ *   s_row = fp16(max|r| / 112), per group q = clamp(ceil(max_group|r| /
+ *   (7 s_row)) - 1, 0, 15), codes against s_row (q + 1) in [-7, 7];
+ *   codes int8 [rows][cols], scale_codes uint8 [rows][cols/group_size]
+ *   (unpacked, 0..15), row_scale fp16 [rows].  cols/group_size <= 1024.
+ * archead_pack_codes: bits 4: two's complement nibbles, byte j of a row =
+ *   columns 2j (low) and 2j+1 (high), [rows][ceil(cols/2)]; bits 5: code j in
+ *   bits 5j..5j+4 of the row's little-endian bit string,
+ *   [rows][ceil(5 cols / 8)] (the canonical layouts of archead_desc).
+ * archead_dequant_symmetric / archead_dequant_residual_sc4: code * scale in
+ *   fp32 (exact), the inverse maps of the two quantisers.
+ * Return ARCHEAD_ERR_INVALID_ARG for shapes that the groups do not divide;
+ * device work is queued on the stream.
+ */
+ARCHEAD_API archead_status archead_quantize_symmetric(const float *x, int64_t rows, int64_t cols, int64_t group_rows,
+                                                      int64_t group_cols, int bits, int8_t *codes, uint16_t *scales,
+                                                      void *stream);
+ARCHEAD_API archead_status archead_quantize_residual_sc4(const float *r, int64_t rows, int64_t cols, int group_size,
+                                                         int8_t *codes, uint8_t *scale_codes, uint16_t *row_scale,
+                                                         void *stream);
+ARCHEAD_API archead_status archead_pack_codes(const int8_t *codes, int64_t rows, int64_t cols, int bits,
+                                              uint8_t *packed, void *stream);
+ARCHEAD_API archead_status archead_dequant_symmetric(const int8_t *codes, const uint16_t *scales, int64_t rows,
+                                                     int64_t cols, int64_t group_rows, int64_t group_cols, float *out,
+                                                     void *stream);
+ARCHEAD_API archead_status archead_dequant_residual_sc4(const int8_t *codes, const uint8_t *scale_codes,
+                                                        const uint16_t *row_scale, int64_t rows, int64_t cols,
+                                                        int group_size, float *out, void *stream);
+
 /* Per-kernel timing with CUDA events on the launch stream (off by default). */
 typedef struct {
   const char *name;  /* static string */

@@ -44,6 +44,8 @@ EXPORTED = (
     "archead_profile_enable", "archead_profile_read", "archead_status_string", "archead_last_error",
     "archead_forward_decode_noalloc", "archead_forward_argmax", "archead_forward_argmax_path",
     "archead_forward_lse_partial", "archead_lse_combine", "archead_argmax_combine",
+    "archead_quantize_symmetric", "archead_quantize_residual_sc4", "archead_pack_codes", "archead_dequant_symmetric",
+    "archead_dequant_residual_sc4",
 )
 
 
@@ -105,6 +107,11 @@ def load() -> ctypes.CDLL:
         "archead_forward_lse_partial": (i32, [vp, vp, i64, vp, i64, vp, i32, vp]),
         "archead_lse_combine": (i32, [vp, i32, i64, vp, vp]),
         "archead_argmax_combine": (i32, [vp, vp, vp, i32, i64, vp, vp, vp]),
+        "archead_quantize_symmetric": (i32, [vp, i64, i64, i64, i64, i32, vp, vp, vp]),
+        "archead_quantize_residual_sc4": (i32, [vp, i64, i64, i32, vp, vp, vp, vp]),
+        "archead_pack_codes": (i32, [vp, i64, i64, i32, vp, vp]),
+        "archead_dequant_symmetric": (i32, [vp, vp, i64, i64, i64, i64, vp, vp]),
+        "archead_dequant_residual_sc4": (i32, [vp, vp, vp, i64, i64, i32, vp, vp]),
         "archead_pack_bytes": (i64, [vp]),
         "archead_device_bytes": (i64, [vp]),
         "archead_debug_dequant": (i32, [vp, i32, i64, i64, vp, vp]),
@@ -260,6 +267,38 @@ def archead_argmax_combine(values, indices, row0, num_shards: int, M: int, index
     """Greedy output from the shards' (value, local index) and their first global rows."""
     _check(load().archead_argmax_combine(_ptr(values), _ptr(indices), _ptr(row0), num_shards, M, _ptr(index),
                                          _ptr(value), _stream_ptr(stream)), "archead_argmax_combine")
+
+
+def archead_quantize_symmetric(x, group_rows: int, group_cols: int, bits: int, codes, scales, stream=None) -> None:
+    """Symmetric quantisation of the fp32 matrix x (rows x cols), one fp16 scale per group block."""
+    rows, cols = x.shape
+    _check(load().archead_quantize_symmetric(_ptr(x), rows, cols, group_rows, group_cols, bits, _ptr(codes),
+                                             _ptr(scales), _stream_ptr(stream)), "archead_quantize_symmetric")
+
+
+def archead_quantize_residual_sc4(r, group_size: int, codes, scale_codes, row_scale, stream=None) -> None:
+    rows, cols = r.shape
+    _check(load().archead_quantize_residual_sc4(_ptr(r), rows, cols, group_size, _ptr(codes), _ptr(scale_codes),
+                                                _ptr(row_scale), _stream_ptr(stream)), "archead_quantize_residual_sc4")
+
+
+def archead_pack_codes(codes, bits: int, packed, stream=None) -> None:
+    rows, cols = codes.shape
+    _check(load().archead_pack_codes(_ptr(codes), rows, cols, bits, _ptr(packed), _stream_ptr(stream)),
+           "archead_pack_codes")
+
+
+def archead_dequant_symmetric(codes, scales, group_rows: int, group_cols: int, out, stream=None) -> None:
+    rows, cols = codes.shape
+    _check(load().archead_dequant_symmetric(_ptr(codes), _ptr(scales), rows, cols, group_rows, group_cols, _ptr(out),
+                                            _stream_ptr(stream)), "archead_dequant_symmetric")
+
+
+def archead_dequant_residual_sc4(codes, scale_codes, row_scale, group_size: int, out, stream=None) -> None:
+    rows, cols = codes.shape
+    _check(load().archead_dequant_residual_sc4(_ptr(codes), _ptr(scale_codes), _ptr(row_scale), rows, cols,
+                                               group_size, _ptr(out), _stream_ptr(stream)),
+           "archead_dequant_residual_sc4")
 
 
 def archead_pack_bytes(pack: Pack) -> int:

@@ -14,4 +14,6 @@ from .inputs import (  # noqa: F401
     make_targets,
     head_nbytes_canonical,
     with_extreme_codes,
+    make_dense_head,
+    make_test_matrix,
 )

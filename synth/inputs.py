@@ -270,6 +270,25 @@ def make_hidden(d: int, M: int, seed: int = 0, n_outliers: int = 4) -> np.ndarra
     return _f32_to_bf16_bits(x.astype(np.float32))
 
 
+def make_dense_head(V: int, D: int, seed: int = 0, rank: int = 64, noise: float = 0.01) -> np.ndarray:
+    """A dense fp32 output head [V, D] standing in for a real one: a
+    rank-`rank` part with singular values log-spaced from 3 down to 0.05 (x
+    0.5), plus i.i.d. Gaussian noise of standard deviation `noise` (the
+    offline construction's input; the real heads are not available)."""
+    s = _streams(seed + 4_000_037, ("u", "v", "noise"))
+    k = min(rank, V, D)
+    U, _ = np.linalg.qr(s["u"].standard_normal((V, k)))
+    Vm, _ = np.linalg.qr(s["v"].standard_normal((D, k)))
+    W = (U * (0.5 * np.geomspace(3.0, 0.05, k))[None, :]) @ Vm.T
+    W += noise * s["noise"].standard_normal((V, D))
+    return W.astype(np.float32)
+
+
+def make_test_matrix(D: int, k: int, seed: int = 0) -> np.ndarray:
+    """Gaussian random test matrix [D, k] for a randomized range finder."""
+    return _streams(seed + 5_000_011, ("omega",))["omega"].standard_normal((D, k))
+
+
 def make_targets(V: int, M: int, seed: int = 0) -> np.ndarray:
     """Next-token targets drawn uniformly over [0, V)."""
     rng = _streams(seed + 2_000_003, ("targets",))["targets"]
