@@ -10,8 +10,9 @@ r_r=32, g=128) at M=1 token (decode); the same line also carries the decode
 sweep M=2..16, the M=4096 prefill (logits and fused cross entropy), a dense
 BF16 cuBLAS head on the same shapes, the batch sweep M=1..8192 through both
 kernels, the same head in the paper's own packed format, the
-Gemma-4-E4B-shaped head, the tiny head (a latency entry beside the oracle)
-and the headline figures of those blocks again as flat top-level keys.
+Gemma-4-E4B-shaped head, the tiny head (a latency entry beside the oracle),
+the offline construction of the Qwen head (Algorithm 1) and the headline
+figures of those blocks again as flat top-level keys.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -402,6 +403,7 @@ def run_ours(args, rank, world, local_rank):
         result["sc4"] = sc4_block(peaks, world, local_rank)
         result["gemma"] = gemma_block(peaks, world, local_rank)
         result["tiny"] = tiny_block(world, local_rank, with_oracle=rank == 0 and world == 1)
+        result["construct"] = construct_block()
         result.update(flat_keys(result))
     if rank == 0 and not args.no_cpu_baseline and world == 1:
         result["cpu_baseline"] = cpu_baseline(wl, x_np, M, budget_s=args.cpu_budget)
@@ -442,6 +444,42 @@ def tiny_block(world, local_rank, with_oracle=True):
     return res
 
 
+def construct_block(N: int = 4096):
+    """Offline construction (Algorithm 1) of the Qwen3-8B-shaped head in the
+    paper's format (r_c=10, r_r=6, g=64, p=0.75, ridge 1e-3) from a seeded
+    dense head and N calibration states, fp32 linear algebra: wall time on the
+    device, and the error left in the activation metric by the realized core
+    and by core plus the unquantised correction, relative to ||W T_p||^2."""
+    import torch
+
+    from paper_2608_02703_gb300 import construct as gc
+    from synth import SHAPES, make_dense_head_device, make_hidden, make_test_matrix
+
+    sh = SHAPES["qwen3-8b-sc4"]
+    W = make_dense_head_device(sh.V, sh.d, seed=0)
+    H = torch.from_numpy(make_hidden(sh.d, N, seed=7).view(np.int16)).cuda().view(torch.bfloat16).float()
+    om_c = torch.from_numpy(make_test_matrix(sh.d, sh.core_rank + 10, seed=1)).cuda().float()
+    om_r = torch.from_numpy(make_test_matrix(sh.d, sh.corr_rank + 10, seed=2)).cuda().float()
+    args = dict(fmt="sc4", omega_core=om_c, omega_corr=om_r, dtype=torch.float32)
+    gc.construct(W[:4096], H, sh.core_rank, sh.corr_rank, sh.group_size, **args)  # warm-up (library load, cuSOLVER)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    head = gc.construct(W, H, sh.core_rank, sh.corr_rank, sh.group_size, keep_intermediates=True, **args)
+    torch.cuda.synchronize()
+    secs = time.perf_counter() - t0
+    T = head["_T"]
+    ref = float(((W @ T) ** 2).sum())
+    e_core = float((head["_E"] @ T).pow(2).sum()) / ref
+    e_corr = float(((head["_E"] - head["_A_w"] @ head["_B_w"]) @ T).pow(2).sum()) / ref
+    res = {"workload": f"qwen3-8b-shaped dense head (V={sh.V}, D={sh.d}), N={N} calibration states, paper's format "
+                       "(r_c=10, r_r=6, g=64), p=0.75, ridge 1e-3, fp32 linear algebra",
+           "seconds": round(secs, 3), "rel_metric_error_core": round(e_core, 6),
+           "rel_metric_error_core_plus_correction": round(e_corr, 6)}
+    del head, W, H
+    torch.cuda.empty_cache()
+    return res
+
+
 def flat_keys(result):
     """The headline numbers of the nested blocks as top-level scalars."""
     out = {}
@@ -463,6 +501,9 @@ def flat_keys(result):
             if mode in bp:
                 out[f"{name}_prefill_m{bp['M']}_{mode}_ms"] = bp[mode]["ms_per_call"]
                 out[f"{name}_prefill_m{bp['M']}_{mode}_frac_bf16_peak"] = bp[mode]["frac_bf16_peak"]
+    c = result.get("construct") or {}
+    if "seconds" in c:
+        out["construct_qwen_sc4_seconds"] = c["seconds"]
     t = result.get("tiny") or {}
     if "us_per_call" in t:
         out["tiny_m4_us"] = t["us_per_call"]

@@ -15,5 +15,6 @@ from .inputs import (  # noqa: F401
     head_nbytes_canonical,
     with_extreme_codes,
     make_dense_head,
+    make_dense_head_device,
     make_test_matrix,
 )

@@ -284,6 +284,24 @@ def make_dense_head(V: int, D: int, seed: int = 0, rank: int = 64, noise: float 
     return W.astype(np.float32)
 
 
+def make_dense_head_device(V: int, D: int, seed: int = 0, rank: int = 64, noise: float = 0.01, device="cuda"):
+    """make_dense_head's recipe drawn on a torch device (fp32), for sizes where
+    a host draw would take long (the full Qwen3-8B-shaped head): the same
+    spectrum and noise level from a seeded torch generator (not the same
+    numbers as make_dense_head)."""
+    import torch
+
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed + 6_000_001)
+    k = min(rank, V, D)
+    U, _ = torch.linalg.qr(torch.randn((V, k), generator=gen, device=device))
+    Vm, _ = torch.linalg.qr(torch.randn((D, k), generator=gen, device=device))
+    s = 0.5 * torch.logspace(np.log10(3.0), np.log10(0.05), k, device=device)
+    W = (U * s[None, :]) @ Vm.T
+    W += noise * torch.randn((V, D), generator=gen, device=device)
+    return W
+
+
 def make_test_matrix(D: int, k: int, seed: int = 0) -> np.ndarray:
     """Gaussian random test matrix [D, k] for a randomized range finder."""
     return _streams(seed + 5_000_011, ("omega",))["omega"].standard_normal((D, k))
