@@ -239,9 +239,12 @@ ARCHEAD_API archead_status archead_argmax_combine(const float *values, const int
 
 /*
  * End-to-end call with HOST buffers: copies x (host, bf16 [M][d]) to the
- * device, runs archead_forward, copies the logits back to logits_host
- * ([M][V], bf16 or fp32) and waits for the stream.  Pinned host memory
- * makes the copies asynchronous with respect to other host work.
+ * device, runs archead_forward into logits_host ([M][V], bf16 or fp32) and
+ * waits for the stream.  When logits_host is pinned and mapped into the
+ * device's address space (cudaHostAlloc / cudaMallocHost, or torch's
+ * pin_memory, under unified addressing) the kernels write the logits into it
+ * directly; otherwise they go to a device buffer owned by the pack and are
+ * copied back.  Either way the call returns with the logits in logits_host.
  */
 ARCHEAD_API archead_status archead_forward_host(archead_pack *pack, const void *x_host, int64_t M, void *logits_host,
                                     archead_out_dtype out_dtype, void *stream);

@@ -549,7 +549,17 @@ archead_status archead_forward_host(archead_pack *pack, const void *x_host, int6
   AH_CUDA(cudaSetDevice(pack->device));
   const size_t xb = (size_t)M * pack->d * 2;
   const size_t yb = (size_t)M * pack->V * (out_dtype == ARCHEAD_OUT_FP32 ? 4 : 2);
-  if (xb > pack->xh_bytes || yb > pack->yh_bytes) {
+  // A pinned, device-mapped output buffer (cudaHostAlloc / cudaMallocHost
+  // under unified addressing) is written by the kernels directly, with no
+  // staging copy; pageable memory goes through a device buffer.
+  void *y_direct = nullptr;
+  cudaPointerAttributes attr{};
+  if (cudaPointerGetAttributes(&attr, logits_host) == cudaSuccess && attr.type == cudaMemoryTypeHost &&
+      attr.devicePointer != nullptr && aligned16(attr.devicePointer))
+    y_direct = attr.devicePointer;
+  cudaGetLastError();  // a pointer the runtime does not know is not an error here
+  const size_t need_y = y_direct ? 0 : yb;
+  if (xb > pack->xh_bytes || need_y > pack->yh_bytes) {
     AH_CUDA(cudaStreamSynchronize(s));
     if (xb > pack->xh_bytes) {
       if (pack->xh_dev) cudaFree(pack->xh_dev), pack->owned_bytes -= (int64_t)pack->xh_bytes;
@@ -559,19 +569,19 @@ archead_status archead_forward_host(archead_pack *pack, const void *x_host, int6
       pack->xh_bytes = xb;
       pack->owned_bytes += (int64_t)xb;
     }
-    if (yb > pack->yh_bytes) {
+    if (need_y > pack->yh_bytes) {
       if (pack->yh_dev) cudaFree(pack->yh_dev), pack->owned_bytes -= (int64_t)pack->yh_bytes;
       pack->yh_dev = nullptr;
       pack->yh_bytes = 0;
-      AH_CUDA(cudaMalloc(&pack->yh_dev, yb));
-      pack->yh_bytes = yb;
-      pack->owned_bytes += (int64_t)yb;
+      AH_CUDA(cudaMalloc(&pack->yh_dev, need_y));
+      pack->yh_bytes = need_y;
+      pack->owned_bytes += (int64_t)need_y;
     }
   }
   AH_CUDA(cudaMemcpyAsync(pack->xh_dev, x_host, xb, cudaMemcpyHostToDevice, s));
-  archead_status st = archead_forward(pack, pack->xh_dev, M, pack->yh_dev, out_dtype, stream);
+  archead_status st = archead_forward(pack, pack->xh_dev, M, y_direct ? y_direct : pack->yh_dev, out_dtype, stream);
   if (st != ARCHEAD_OK) return st;
-  AH_CUDA(cudaMemcpyAsync(logits_host, pack->yh_dev, yb, cudaMemcpyDeviceToHost, s));
+  if (!y_direct) AH_CUDA(cudaMemcpyAsync(logits_host, pack->yh_dev, yb, cudaMemcpyDeviceToHost, s));
   AH_CUDA(cudaStreamSynchronize(s));
   return ARCHEAD_OK;
 }

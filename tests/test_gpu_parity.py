@@ -231,17 +231,25 @@ def test_zero_tokens_is_a_no_op():
     assert archead.archead_sync_status(pack) == archead.OK
 
 
-def test_forward_host_matches_device():
+@pytest.mark.parametrize("M", [4, 300])
+def test_forward_host_matches_device(M):
+    """Host buffers: pinned (the kernels write the output in place) and
+    pageable (staged through the pack's device buffer), bit for bit the
+    device-buffer forward, on the decode and the prefill kernel."""
     import torch
 
     pack, head = get("tiny")
     shape = SHAPES["tiny"]
-    x = make_hidden(shape.d, 4, seed=9)
-    dev = gu.forward(pack, x, archead.OUT_BF16)
-    xh = torch.from_numpy(x.view(np.int16)).pin_memory()
-    yh = torch.empty((4, shape.V), dtype=torch.bfloat16).pin_memory()
-    archead.archead_forward_host(pack, xh, 4, yh, archead.OUT_BF16)
-    assert np.array_equal(yh.float().numpy().astype(np.float64), dev)
+    x = make_hidden(shape.d, M, seed=9)
+    for dt, out in ((torch.bfloat16, archead.OUT_BF16), (torch.float32, archead.OUT_FP32)):
+        dev = gu.forward(pack, x, out)
+        xh = torch.from_numpy(x.view(np.int16)).pin_memory()
+        yh = torch.full((M, shape.V), float("nan"), dtype=dt).pin_memory()
+        archead.archead_forward_host(pack, xh, M, yh, out)
+        assert np.array_equal(yh.float().numpy().astype(np.float64), dev)
+        yp = torch.full((M, shape.V), float("nan"), dtype=dt)  # pageable
+        archead.archead_forward_host(pack, torch.from_numpy(x.view(np.int16).copy()), M, yp, out)
+        assert np.array_equal(yp.float().numpy().astype(np.float64), dev)
 
 
 def test_wait_timeout_is_reported_and_recoverable():
