@@ -25,6 +25,7 @@
 // accumulator block promoted once by s_row: no per-group hand-back.
 #pragma once
 
+#include <cfloat>
 #include <cuda.h>
 
 #include "device.cuh"
@@ -41,6 +42,8 @@ constexpr int kPfStageBytes = kPfABytes + kPfBBytes + kPfCodeBytes;
 constexpr int kPfThreads = 512;
 constexpr int kPfTmemCols = 512;                  // two 256-column accumulators
 constexpr int kPfSmem = 1024 + kPfStages * kPfStageBytes + 256;
+constexpr float kLog2e = 1.4426950408889634f;  // log2(e)
+constexpr float kLn2 = 0.6931471805599453f;    // ln(2)
 
 struct PrefillParams {
   CUtensorMap tmap_x;   // bf16 [M][d], box 64 x 128, 128B swizzle
@@ -110,6 +113,28 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 16 lanes x 32 columns starting at taddr (lane field = first lane) in the
+// 16x256b shape, 4 repetitions of 8 columns: in repetition c thread t holds
+// v[4c + j] = (lane t/4 + 8 (j >> 1), column 8c + 2 (t % 4) + (j & 1)).
+__device__ __forceinline__ void tmem_ld16x256b_x4(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x256b.x4.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// 2^x by the special-function unit (ex2.approx, flushes denormal results).
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;\n" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // d0 += a * b0 and d1 += a * b1 as one packed fp32x2 FMA (round to nearest).
 __device__ __forceinline__ void fma2(float &d0, float &d1, float a, float b0, float b1) {
   asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %2};\n mov.b64 rb, {%3, %4};\n mov.b64 rd, {%0, %1};\n"
@@ -118,12 +143,15 @@ __device__ __forceinline__ void fma2(float &d0, float &d1, float a, float b0, fl
       : "f"(a), "f"(b0), "f"(b1));
 }
 
-// One step of the log-sum-exp merge: (m, s) of two disjoint sets -> of their union.
-__device__ __forceinline__ void lse_pair_merge(float am, float as, float bm, float bs, float &m, float &s) {
-  const float mx = fmaxf(am, bm), mn = fminf(am, bm);
-  const float e = mn == -INFINITY ? 0.f : __expf(mn - mx);
-  s = am >= bm ? fmaf(bs, e, as) : fmaf(as, e, bs);
-  m = mx;
+// One step of the base-2 log-sum-exp merge: (m, s) of two disjoint sets, s
+// the sum of 2^(y - m), -> (m, s) of their union.  Maxima are finite: rows
+// past the vocabulary enter as -FLT_MAX, whose difference with itself is 0
+// and with any logit rounds to +-FLT_MAX or +-inf (weight 0).
+__device__ __forceinline__ void lse2_merge(float am, float as, float bm, float bs, float &m, float &s) {
+  const float d = am - bm;
+  const float e = ex2_approx(-fabsf(d));
+  s = d >= 0.f ? fmaf(bs, e, as) : fmaf(as, e, bs);
+  m = fmaxf(am, bm);
 }
 
 // Shared-memory matrix descriptor: K-major operand in the 128-byte swizzle
@@ -218,13 +246,17 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   bool mma_leader = false;  // the lane of warp 1 that issues the MMAs
 
   // Registers are rebalanced between warpgroups (launch: 512 x 128): the
-  // producer/MMA warpgroup and the converters keep 88 each, the two promotion
-  // warpgroups get 168 each (128 fp32 accumulators per thread):
-  // 4*32*(88 + 88) + 8*32*168 = 65536.  Each role's code follows its own
-  // setmaxnreg so that the compiler allocates within that budget; this split
-  // is the one that compiles without spills.
+  // converters keep 88, the producer/MMA warpgroup 88 (logits, greedy) or 56
+  // (cross entropy), the two promotion warpgroups get the rest, 168 or 184
+  // (128 fp32 accumulators per thread; the cross-entropy epilogue needs
+  // more): 4*32*(88 + 88) + 8*32*168 = 4*32*(56 + 88) + 8*32*184 = 65536.
+  // Each role's code follows its own setmaxnreg so that the compiler
+  // allocates within that budget; these splits compile without spills.
   if (warp < 4) {
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 88;\n" ::: "memory");
+    if constexpr (kMode == 1)
+      asm volatile("setmaxnreg.dec.sync.aligned.u32 56;\n" ::: "memory");
+    else
+      asm volatile("setmaxnreg.dec.sync.aligned.u32 88;\n" ::: "memory");
   if (warp == 0) {
     // ------------------------------ producer ------------------------------
     // The whole warp runs the loop (uniform waits); one elected lane issues.
@@ -391,11 +423,18 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     }
   } else {
     // ------------------------------ promotion + epilogue ------------------------------
-    asm volatile("setmaxnreg.inc.sync.aligned.u32 168;\n" ::: "memory");
+    if constexpr (kMode == 1)
+      asm volatile("setmaxnreg.inc.sync.aligned.u32 184;\n" ::: "memory");
+    else
+      asm volatile("setmaxnreg.inc.sync.aligned.u32 168;\n" ::: "memory");
     const int pw = warp - 8;
     const int lg = pw & 3;            // TMEM lane group (rows 32*lg .. 32*lg+31)
     const int ch = pw >> 2;           // column half (tokens 128*ch .. 128*ch+127)
     const int r_in_tile = lg * 32 + lane;
+    // Cross entropy reads TMEM in the 16x256b shape (4 rows x 32 tokens per
+    // thread) and accumulates in base 2 (factors times log2 e); logits and
+    // greedy read 32x32b (one row x 128 tokens per thread).
+    constexpr bool kQuad = kMode == 1;
     int bcount = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
       const int vt = t / p.num_mt, mt = t % p.num_mt;
@@ -406,22 +445,54 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
       for (int i = 0; i < 128; ++i) acc[i] = 0.f;
       const int nb = bp.nblocks();
       for (int b = 0; b < nb; ++b) {
-        float f;
-        if (b < bp.nres)
-          f = kSC4 ? fp16_bits_to_f32(p.s_row[row])
-                    : fp16_bits_to_f32(p.scales[((int64_t)vt * p.G_pad + b) * kTileRows + r_in_tile]);
-        else if (b == bp.nres && bp.core_sub > 0) f = 1.f;
-        else f = fp16_bits_to_f32(p.s_a[row]);
+        // Promotion factor of block b for the thread's row(s) of the tile.
+        float f[kQuad ? 4 : 1];
+        if constexpr (kQuad) {
+          // Rows lane / 4 + 8k of the warp's 32: one base pointer, offsets 8k.
+          const int rt0 = lg * 32 + (lane >> 2);
+          const uint16_t *fs = nullptr;
+          if (b < bp.nres)
+            fs = kSC4 ? p.s_row + (int64_t)vt * kTileRows + rt0
+                      : p.scales + ((int64_t)vt * p.G_pad + b) * kTileRows + rt0;
+          else if (!(b == bp.nres && bp.core_sub > 0)) fs = p.s_a + (int64_t)vt * kTileRows + rt0;
+#pragma unroll
+          for (int k = 0; k < 4; ++k) f[k] = fs ? fp16_bits_to_f32(fs[8 * k]) * kLog2e : kLog2e;
+        } else {
+          if (b < bp.nres)
+            f[0] = kSC4 ? fp16_bits_to_f32(p.s_row[row])
+                        : fp16_bits_to_f32(p.scales[((int64_t)vt * p.G_pad + b) * kTileRows + r_in_tile]);
+          else if (b == bp.nres && bp.core_sub > 0) f[0] = 1.f;
+          else f[0] = fp16_bits_to_f32(p.s_a[row]);
+        }
         const int buf = bcount & 1;
         if (!mbar_wait_warp(&acc_full[buf], (bcount >> 1) & 1, p.wait_budget, abort_flag, p.err)) goto done;
         tc_fence_after();
         const uint32_t taddr = tmem_base + ((uint32_t)(lg * 32) << 16) + buf * kPfN + ch * 128;
+        if constexpr (kQuad) {
+          // acc[64h + 4kk + j] = row 8 (2h + (j >> 1)) + lane / 4 of the warp's
+          // 32, token column 8kk + 2 (lane % 4) + (j & 1), kk = 0..15.
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          float v[32];
-          tmem_ld32(taddr + c * 32, v);
+          for (int h = 0; h < 2; ++h) {
 #pragma unroll
-          for (int i = 0; i < 32; i += 2) fma2(acc[c * 32 + i], acc[c * 32 + i + 1], f, v[i], v[i + 1]);
+            for (int cc = 0; cc < 4; ++cc) {
+              float v[16];
+              tmem_ld16x256b_x4(taddr + ((uint32_t)(16 * h) << 16) + cc * 32, v);
+              float *a = acc + 64 * h + 16 * cc;
+#pragma unroll
+              for (int c = 0; c < 4; ++c) {
+                fma2(a[4 * c], a[4 * c + 1], f[2 * h], v[4 * c], v[4 * c + 1]);
+                fma2(a[4 * c + 2], a[4 * c + 3], f[2 * h + 1], v[4 * c + 2], v[4 * c + 3]);
+              }
+            }
+          }
+        } else {
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            float v[32];
+            tmem_ld32(taddr + c * 32, v);
+#pragma unroll
+            for (int i = 0; i < 32; i += 2) fma2(acc[c * 32 + i], acc[c * 32 + i + 1], f[0], v[i], v[i + 1]);
+          }
         }
         tc_fence_before();
         __syncwarp();
@@ -446,8 +517,8 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
         }
       } else if (kMode == 2) {
         // Greedy partials: the largest logit of each token over the warp's 32
-        // rows and its row (the lowest on ties), by the same token-halving
-        // butterfly as the cross entropy below: values in acc[0..63], rows
+        // rows and its row (the lowest on ties), by a butterfly that halves
+        // the token set per step (lane offsets 16 .. 1): values in acc[0..63], rows
         // (int bits) in acc[64..127]; lane L ends with tokens 4L..4L+3.
         const int64_t rowbase = row - lane;
         if (row >= p.V) {
@@ -489,61 +560,77 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
           if (m < p.M) p.ce_part[((int64_t)vt * 4 + lg) * p.M + m] = make_float2(acc[j], acc[64 + j]);
         }
       } else {
+        // Layout (see the promotion): this thread holds rows rbase + ru + 8 kr
+        // (kr = 0..3) of 32 token columns col(k) = 8 (k >> 1) + 2 cq + (k & 1),
+        // k = 0..31, row kr of column k at acc[i0(k) + {0, 2, 64, 66}[kr]].
+        const int64_t rbase = (int64_t)vt * kTileRows + lg * 32;
+        const int ru = lane >> 2, cq = lane & 3;
         // Target logits first: a token whose target is one of this warp's 32
-        // rows takes its value from the owning lane (rare: about one token in
-        // 37 per warp and tile, so the slow path is a warp-uniform branch).
-        const int64_t rowbase = row - lane;
+        // rows takes its value from the thread holding it (rare: about one
+        // token in 37 per warp and tile, so the slow path is a warp-uniform
+        // branch).  Lane (ru, cq) reads the targets of the columns it ends
+        // with: 16 ru + 8 (j >> 1) + 2 cq + (j & 1), j = 0..3.
         int tg[4];
         bool hit = false;
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          const int m = m0 + 4 * lane + j;
-          tg[j] = m < p.M ? p.targets[m] - p.row0 : -1;  // this pack's row numbering
-          hit |= tg[j] >= rowbase && tg[j] < rowbase + 32;
+          const int m = m0 + 16 * ru + 8 * (j >> 1) + 2 * cq + (j & 1);
+          const int64_t t64 = m < p.M ? (int64_t)p.targets[m] - p.row0 - rbase : -1;  // row within the warp's 32
+          tg[j] = t64 >= 0 && t64 < 32 ? (int)t64 : -1;
+          hit |= tg[j] >= 0;
         }
         if (__any_sync(0xffffffffu, hit)) {
 #pragma unroll
-          for (int k = 0; k < 128; ++k) {
-            const int tk = __shfl_sync(0xffffffffu, tg[k & 3], k >> 2);
-            const float val = __shfl_sync(0xffffffffu, acc[k], (int)((tk - rowbase) & 31));
-            if (lane == (k >> 2) && tk >= rowbase && tk < rowbase + 32) p.ce_tlogit[m0 + k] = val;
+          for (int col = 0; col < 128; ++col) {
+            const int j = 2 * ((col >> 3) & 1) + (col & 1);
+            const int owner = 4 * (col >> 4) + ((col >> 1) & 3);  // lane that read this column's target
+            const int r = __shfl_sync(0xffffffffu, tg[j], owner);
+            if (r >= 0) {  // warp-uniform
+              const int i0 = 4 * (col >> 3) + (col & 1);
+              const float mine = r & 16 ? (r & 8 ? acc[i0 + 66] : acc[i0 + 64]) : (r & 8 ? acc[i0 + 2] : acc[i0]);
+              const float v = __shfl_sync(0xffffffffu, mine, 4 * (r & 7) + ((col >> 1) & 3));
+              if (lane == owner) p.ce_tlogit[m0 + col] = v * kLn2;
+            }
           }
         }
-        // (max, sum of exp) over the warp's 32 rows for each of the 128
-        // tokens, by a butterfly that halves the token set per step: in the
-        // step with lane offset o the lane with bit o set keeps the upper
-        // half and merges the partner's copy of it.  After the five steps
-        // lane L holds tokens 4L..4L+3.  Maxima live in acc[0..63], sums in
-        // acc[64..127]; rows past V enter as -inf.
-        if (row >= p.V) {
+        // Rows past V (last tile only) enter as -FLT_MAX: weight 0 against any
+        // logit, and a finite (max, count) when the warp holds no real row.
+        if (rbase + 32 > p.V) {
 #pragma unroll
-          for (int i = 0; i < 128; ++i) acc[i] = -INFINITY;
-        }
-        {
-          const bool up = lane & 16;
-#pragma unroll
-          for (int j = 0; j < 64; ++j) {
-            const float keep = up ? acc[j + 64] : acc[j];
-            const float give = up ? acc[j] : acc[j + 64];
-            const float recv = __shfl_xor_sync(0xffffffffu, give, 16);
-            lse_pair_merge(keep, 1.f, recv, 1.f, acc[j], acc[64 + j]);
+          for (int i = 0; i < 128; ++i) {
+            const int kr = 2 * (i >> 6) + ((i >> 1) & 1);
+            if (rbase + ru + 8 * kr >= p.V) acc[i] = -FLT_MAX;
           }
         }
+        // (max, sum of 2^(y - max)) of each column over the thread's 4 rows...
+        float mx[32], sm[32];
 #pragma unroll
-        for (int n = 64, o = 8; n > 4; n >>= 1, o >>= 1) {
+        for (int k = 0; k < 32; ++k) {
+          const int i0 = 4 * (k >> 1) + (k & 1);
+          const float v0 = acc[i0], v1 = acc[i0 + 2], v2 = acc[i0 + 64], v3 = acc[i0 + 66];
+          const float mk = fmaxf(fmaxf(v0, v1), fmaxf(v2, v3));
+          mx[k] = mk;
+          sm[k] = (ex2_approx(v0 - mk) + ex2_approx(v1 - mk)) + (ex2_approx(v2 - mk) + ex2_approx(v3 - mk));
+        }
+        // ...then over the 8 lanes with the same lane % 4 (lane bits 4, 3, 2)
+        // by a butterfly that halves the column set per step: the lane with
+        // bit o set keeps the upper half and merges the partner's copy of it.
+        // Lane (ru, cq) ends with k = 4 ru + j, j = 0..3.
+#pragma unroll
+        for (int n = 32, o = 16; n > 4; n >>= 1, o >>= 1) {
           const bool up = lane & o;
 #pragma unroll
           for (int j = 0; j < n / 2; ++j) {
-            const float km = up ? acc[j + n / 2] : acc[j], ks = up ? acc[64 + j + n / 2] : acc[64 + j];
-            const float gm = up ? acc[j] : acc[j + n / 2], gs = up ? acc[64 + j] : acc[64 + j + n / 2];
+            const float km = up ? mx[j + n / 2] : mx[j], ks = up ? sm[j + n / 2] : sm[j];
+            const float gm = up ? mx[j] : mx[j + n / 2], gs = up ? sm[j] : sm[j + n / 2];
             const float rm = __shfl_xor_sync(0xffffffffu, gm, o), rs = __shfl_xor_sync(0xffffffffu, gs, o);
-            lse_pair_merge(km, ks, rm, rs, acc[j], acc[64 + j]);
+            lse2_merge(km, ks, rm, rs, mx[j], sm[j]);
           }
         }
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          const int m = m0 + 4 * lane + j;
-          if (m < p.M) p.ce_part[((int64_t)vt * 4 + lg) * p.M + m] = make_float2(acc[j], acc[64 + j]);
+          const int m = m0 + 16 * ru + 8 * (j >> 1) + 2 * cq + (j & 1);
+          if (m < p.M) p.ce_part[((int64_t)vt * 4 + lg) * p.M + m] = make_float2(mx[j] * kLn2, sm[j]);
         }
       }
     }
