@@ -252,6 +252,31 @@ def test_forward_host_matches_device(M):
         assert np.array_equal(yp.float().numpy().astype(np.float64), dev)
 
 
+def test_forward_host_repeated_calls_with_new_inputs():
+    """Repeated host calls on the same pinned buffers: every call must read
+    the buffers' current contents and match the device-buffer forward bit
+    for bit, also after M changes and after the pack's workspace is
+    reallocated by a larger forward in between."""
+    import torch
+
+    pack, head = get("ragged")
+    shape = SHAPES["ragged"]
+    for M in (3, 16, 3):
+        xh = torch.empty((M, shape.d), dtype=torch.int16).pin_memory()
+        yh = torch.empty((M, shape.V), dtype=torch.bfloat16).pin_memory()
+        for call in range(5):
+            x = make_hidden(shape.d, M, seed=40 + 7 * M + call)
+            xh.copy_(torch.from_numpy(x.view(np.int16)))
+            yh.fill_(float("nan"))
+            archead.archead_forward_host(pack, xh, M, yh, archead.OUT_BF16)
+            dev = gu.forward(pack, x, archead.OUT_BF16)
+            assert np.array_equal(yh.float().numpy().astype(np.float64), dev), f"M={M} call {call}"
+            if call == 2:  # a larger forward grows the workspace between two replays
+                big = make_hidden(shape.d, 600, seed=5)
+                gu.forward(pack, big, archead.OUT_BF16)
+    assert archead.archead_sync_status(pack) == archead.OK
+
+
 def test_wait_timeout_is_reported_and_recoverable():
     pack, head = get("ragged")
     archead.archead_set_wait_budget(pack, 20_000)  # cycles: a few microseconds
