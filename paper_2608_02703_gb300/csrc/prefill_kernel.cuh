@@ -23,6 +23,13 @@
 // 4-bit code q.  The converters fold q + 1 into the operand (code * (q + 1)
 // stays an exact bf16 integer, |.| <= 128), so the whole residual is one
 // accumulator block promoted once by s_row: no per-group hand-back.
+//
+// Epilogues: logits (each promotion thread stores one row of its 128 tokens),
+// greedy partials (largest logit and its row per token over each warp's 32
+// rows) and cross-entropy partials (max and sum of exp per token over each
+// warp's 32 rows, plus the target's logit).  The cross-entropy instance
+// reads TMEM in the 16x256b shape, so that a thread holds 4 rows of 32
+// tokens and most of the log-sum-exp is thread-local.
 #pragma once
 
 #include <cfloat>
