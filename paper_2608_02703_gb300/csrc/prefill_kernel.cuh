@@ -27,9 +27,9 @@
 // Epilogues: logits (each promotion thread stores one row of its 128 tokens),
 // greedy partials (largest logit and its row per token over each warp's 32
 // rows) and cross-entropy partials (max and sum of exp per token over each
-// warp's 32 rows, plus the target's logit).  The cross-entropy instance
-// reads TMEM in the 16x256b shape, so that a thread holds 4 rows of 32
-// tokens and most of the log-sum-exp is thread-local.
+// warp's 32 rows, plus the target's logit).  The cross-entropy and greedy
+// instances read TMEM in the 16x256b shape, so that a thread holds 4 rows
+// of 32 tokens and most of the reduction over rows is thread-local.
 #pragma once
 
 #include <cfloat>
@@ -253,14 +253,13 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   bool mma_leader = false;  // the lane of warp 1 that issues the MMAs
 
   // Registers are rebalanced between warpgroups (launch: 512 x 128): the
-  // converters keep 88, the producer/MMA warpgroup 88 (logits, greedy) or 56
-  // (cross entropy), the two promotion warpgroups get the rest, 168 or 184
-  // (128 fp32 accumulators per thread; the cross-entropy epilogue needs
-  // more): 4*32*(88 + 88) + 8*32*168 = 4*32*(56 + 88) + 8*32*184 = 65536.
+  // converters keep 88, the producer/MMA warpgroup 88 (logits) or 56 (cross
+  // entropy, greedy), the two promotion warpgroups get the rest, 168 or 184
+  // (128 fp32 accumulators per thread; the 4-row epilogues need more): 4*32*(88 + 88) + 8*32*168 = 4*32*(56 + 88) + 8*32*184 = 65536.
   // Each role's code follows its own setmaxnreg so that the compiler
   // allocates within that budget; these splits compile without spills.
   if (warp < 4) {
-    if constexpr (kMode == 1)
+    if constexpr (kMode != 0)
       asm volatile("setmaxnreg.dec.sync.aligned.u32 56;\n" ::: "memory");
     else
       asm volatile("setmaxnreg.dec.sync.aligned.u32 88;\n" ::: "memory");
@@ -430,7 +429,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     }
   } else {
     // ------------------------------ promotion + epilogue ------------------------------
-    if constexpr (kMode == 1)
+    if constexpr (kMode != 0)
       asm volatile("setmaxnreg.inc.sync.aligned.u32 184;\n" ::: "memory");
     else
       asm volatile("setmaxnreg.inc.sync.aligned.u32 168;\n" ::: "memory");
@@ -438,10 +437,10 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     const int lg = pw & 3;            // TMEM lane group (rows 32*lg .. 32*lg+31)
     const int ch = pw >> 2;           // column half (tokens 128*ch .. 128*ch+127)
     const int r_in_tile = lg * 32 + lane;
-    // Cross entropy reads TMEM in the 16x256b shape (4 rows x 32 tokens per
-    // thread) and accumulates in base 2 (factors times log2 e); logits and
-    // greedy read 32x32b (one row x 128 tokens per thread).
-    constexpr bool kQuad = kMode == 1;
+    // Cross entropy and greedy read TMEM in the 16x256b shape (4 rows x 32
+    // tokens per thread; cross entropy accumulates in base 2, its factors
+    // times log2 e); logits read 32x32b (one row x 128 tokens per thread).
+    constexpr bool kQuad = kMode != 0;
     int bcount = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
       const int vt = t / p.num_mt, mt = t % p.num_mt;
@@ -463,7 +462,10 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
                       : p.scales + ((int64_t)vt * p.G_pad + b) * kTileRows + rt0;
           else if (!(b == bp.nres && bp.core_sub > 0)) fs = p.s_a + (int64_t)vt * kTileRows + rt0;
 #pragma unroll
-          for (int k = 0; k < 4; ++k) f[k] = fs ? fp16_bits_to_f32(fs[8 * k]) * kLog2e : kLog2e;
+          for (int k = 0; k < 4; ++k) {
+            f[k] = fs ? fp16_bits_to_f32(fs[8 * k]) : 1.f;
+            if (kMode == 1) f[k] *= kLog2e;
+          }
         } else {
           if (b < bp.nres)
             f[0] = kSC4 ? fp16_bits_to_f32(p.s_row[row])
@@ -524,47 +526,54 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
         }
       } else if (kMode == 2) {
         // Greedy partials: the largest logit of each token over the warp's 32
-        // rows and its row (the lowest on ties), by a butterfly that halves
-        // the token set per step (lane offsets 16 .. 1): values in acc[0..63], rows
-        // (int bits) in acc[64..127]; lane L ends with tokens 4L..4L+3.
-        const int64_t rowbase = row - lane;
-        if (row >= p.V) {
+        // rows and its row (the lowest on ties).  Layout as for the cross
+        // entropy below: rows rbase + ru + 8 kr of the 32 token columns
+        // col(k) = 8 (k >> 1) + 2 cq + (k & 1); first over the thread's 4
+        // rows (ascending, so the first maximum wins), then a butterfly over
+        // lane bits 4, 3, 2 that halves the column set per step.
+        const int rbase = vt * kTileRows + lg * 32;
+        const int ru = lane >> 2, cq = lane & 3;
+        if (rbase + 32 > p.V) {
 #pragma unroll
-          for (int i = 0; i < 128; ++i) acc[i] = -INFINITY;
-        }
-        {
-          const bool up = lane & 16;
-          const int my_row = (int)row, partner_row = (int)(rowbase + (lane ^ 16));
-#pragma unroll
-          for (int j = 0; j < 64; ++j) {
-            const float keep = up ? acc[j + 64] : acc[j];
-            const float give = up ? acc[j] : acc[j + 64];
-            const float recv = __shfl_xor_sync(0xffffffffu, give, 16);
-            const bool take = recv > keep || (recv == keep && partner_row < my_row);
-            acc[j] = take ? recv : keep;
-            acc[64 + j] = __int_as_float(take ? partner_row : my_row);
+          for (int i = 0; i < 128; ++i) {
+            const int kr = 2 * (i >> 6) + ((i >> 1) & 1);
+            if (rbase + ru + 8 * kr >= p.V) acc[i] = -INFINITY;
           }
         }
+        float bv[32];
+        int bi[32];
 #pragma unroll
-        for (int n = 64, o = 8; n > 4; n >>= 1, o >>= 1) {
+        for (int k = 0; k < 32; ++k) {
+          const int i0 = 4 * (k >> 1) + (k & 1);
+          const int r = rbase + ru;
+          float v = acc[i0];
+          int ix = r;
+          if (acc[i0 + 2] > v) v = acc[i0 + 2], ix = r + 8;
+          if (acc[i0 + 64] > v) v = acc[i0 + 64], ix = r + 16;
+          if (acc[i0 + 66] > v) v = acc[i0 + 66], ix = r + 24;
+          bv[k] = v;
+          bi[k] = ix;
+        }
+#pragma unroll
+        for (int n = 32, o = 16; n > 4; n >>= 1, o >>= 1) {
           const bool up = lane & o;
 #pragma unroll
           for (int j = 0; j < n / 2; ++j) {
-            const float kv = up ? acc[j + n / 2] : acc[j];
-            const int ki = __float_as_int(up ? acc[64 + j + n / 2] : acc[64 + j]);
-            const float gv = up ? acc[j] : acc[j + n / 2];
-            const float gi = up ? acc[64 + j] : acc[64 + j + n / 2];
+            const float kv = up ? bv[j + n / 2] : bv[j];
+            const int ki = up ? bi[j + n / 2] : bi[j];
+            const float gv = up ? bv[j] : bv[j + n / 2];
+            const int gi = up ? bi[j] : bi[j + n / 2];
             const float rv = __shfl_xor_sync(0xffffffffu, gv, o);
-            const int ri = __float_as_int(__shfl_xor_sync(0xffffffffu, gi, o));
+            const int ri = __shfl_xor_sync(0xffffffffu, gi, o);
             const bool take = rv > kv || (rv == kv && ri < ki);
-            acc[j] = take ? rv : kv;
-            acc[64 + j] = __int_as_float(take ? ri : ki);
+            bv[j] = take ? rv : kv;
+            bi[j] = take ? ri : ki;
           }
         }
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          const int m = m0 + 4 * lane + j;
-          if (m < p.M) p.ce_part[((int64_t)vt * 4 + lg) * p.M + m] = make_float2(acc[j], acc[64 + j]);
+          const int m = m0 + 16 * ru + 8 * (j >> 1) + 2 * cq + (j & 1);
+          if (m < p.M) p.ce_part[((int64_t)vt * 4 + lg) * p.M + m] = make_float2(bv[j], __int_as_float(bi[j]));
         }
       } else {
         // Layout (see the promotion): this thread holds rows rbase + ru + 8 kr
