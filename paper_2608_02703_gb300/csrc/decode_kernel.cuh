@@ -111,6 +111,19 @@ static DecodePlan decode_plan(int d_pad, int nls, int g, int M, int variant) {
   return pl;
 }
 
+// ldmatrix: four (two) 8x8 b16 matrices; lane L gives the address of row
+// L % 8 of matrix L / 8.  Thread t receives row t / 4, elements 2 (t % 4) and
+// 2 (t % 4) + 1 of each: the m16n8k16 B fragment when the rows are tokens
+// and the 8 elements k values.
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t &r0, uint32_t &r1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];\n" : "=r"(r0), "=r"(r1) : "r"(addr));
+}
+
 // acc += f_lo * part (rows gq) and f_hi * part (rows gq + 8).
 template <int NT>
 __device__ __forceinline__ void promote(float (&acc)[NT][4], const float (&part)[NT][4], float f_lo, float f_hi) {
@@ -364,6 +377,9 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
   const uint16_t *xb[NT];
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) xb[nt] = kStreamX ? nullptr : xs_s + min(8 * nt + gq, p.M - 1) * xrow + 2 * cq;
+  // ldmatrix row address of this lane (one token tile): token L % 8 (clamped
+  // to the M rows held), k offset 8 (L / 8) % 2.
+  const uint16_t *xl = kStreamX || !kSC4 ? nullptr : xs_s + min(lane & 7, p.M - 1) * xrow + 8 * ((lane >> 3) & 1);
   bool t_ready = false;
 
   int st = 0;     // ring slot
@@ -445,18 +461,32 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
         for (int j = 0; j < 4; ++j) {
           const int ks = c * 4 + j;  // k step within the stage
           uint32_t b[NT][2];
+          if constexpr (kStreamX && NT == 2) {
+            // Matrices (tokens 0-7 | 8-15) x (k 0-7 | 8-15) of the k step: lane
+            // L addresses token 8 (L / 16) + L % 8 at 16-byte chunk 2j + (L / 8) % 2
+            // of its 128-byte row (chunk index XOR token % 8).
+            const int tok = 8 * (lane >> 4) + (lane & 7);
+            ldsm_x4(smem_u32(sbuf + Geom::kXOff + c * kXChunkBytes + tok * 128 +
+                             (((2 * j + ((lane >> 3) & 1)) ^ (tok & 7)) << 4)),
+                    b[0][0], b[0][1], b[1][0], b[1][1]);
+          } else if constexpr (!kStreamX && NT == 1 && kSC4) {
+            // Tokens 0-7 (clamped to M) x (k 0-7 | 8-15) of the k step.  (The
+            // INT8 format's resident instance keeps its two 32-bit loads: its
+            // whole forward measured 0.4 us slower with ldmatrix here, the SC4
+            // instance's 1.2 us faster.)
+            ldsm_x2(smem_u32(xl + kbase + ks * 16), b[0][0], b[0][1]);
+          } else {
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
-            if (kStreamX) {
-              // Token 8*nt + gq, k = 16*ks + 2*cq (+8): 128-byte rows, 16-byte
-              // chunk index XOR (row % 8) = gq.
-              const uint8_t *xr = sbuf + Geom::kXOff + c * kXChunkBytes + (8 * nt + gq) * 128 + 4 * cq;
-              b[nt][0] = *reinterpret_cast<const uint32_t *>(xr + (((2 * j) ^ gq) << 4));
-              b[nt][1] = *reinterpret_cast<const uint32_t *>(xr + (((2 * j + 1) ^ gq) << 4));
-            } else {
-              const uint16_t *q = xb[nt] + kbase + ks * 16;
-              b[nt][0] = *reinterpret_cast<const uint32_t *>(q);
-              b[nt][1] = *reinterpret_cast<const uint32_t *>(q + 8);
+            for (int nt = 0; nt < NT; ++nt) {
+              if (kStreamX) {
+                const uint8_t *xr = sbuf + Geom::kXOff + c * kXChunkBytes + (8 * nt + gq) * 128 + 4 * cq;
+                b[nt][0] = *reinterpret_cast<const uint32_t *>(xr + (((2 * j) ^ gq) << 4));
+                b[nt][1] = *reinterpret_cast<const uint32_t *>(xr + (((2 * j + 1) ^ gq) << 4));
+              } else {
+                const uint16_t *q = xb[nt] + kbase + ks * 16;
+                b[nt][0] = *reinterpret_cast<const uint32_t *>(q);
+                b[nt][1] = *reinterpret_cast<const uint32_t *>(q + 8);
+              }
             }
           }
           // First k step of a group (compile-time when groups fit in a stage).
