@@ -70,10 +70,13 @@ typedef enum {
 } archead_format;
 
 typedef enum {
-  ARCHEAD_PATH_AUTO = 0,    /* decode kernel for M <= 48, prefill kernel above (and for
-                               heads too wide for the decode kernel's shared memory)  */
-  ARCHEAD_PATH_DECODE = 1,  /* memory-bound decode kernel (tokens taken 16 at a time);
-                               ARCHEAD_ERR_UNSUPPORTED for heads too wide for it     */
+  ARCHEAD_PATH_AUTO = 0,    /* decode kernel for M <= 64 (M <= 48 for heads whose
+                               shared memory leaves only 16-token launches), prefill
+                               kernel above (and for heads too wide for the decode
+                               kernel's shared memory)                                 */
+  ARCHEAD_PATH_DECODE = 1,  /* decode kernel: one launch per 16, 32 or 64 tokens (by M
+                               and the head's width); ARCHEAD_ERR_UNSUPPORTED for
+                               heads too wide for it                                   */
   ARCHEAD_PATH_PREFILL = 2  /* tensor-core prefill kernel                               */
 } archead_path;
 

@@ -109,18 +109,23 @@ cudaError_t ensure_counters(archead_pack *p, int n, cudaStream_t s) {
 
 struct ForwardPlan {
   size_t partial_off = 0, ts_off = 0, ce_part_off = 0, tlogit_off = 0, total = 0;
-  int nchunks = 0;
+  int variant = 0, chunk_tokens = 0, nchunks = 0;
 };
 
-// Lay out the workspace of one forward over M tokens on the decode path.
+// Lay out the workspace of one forward over M tokens on the decode path: one
+// kernel instance for every launch (so that the cross-entropy partial blocks
+// have one layout), chunks of as many tokens as it takes.
 ForwardPlan plan_decode(archead_pack *p, int64_t M, bool ce) {
   ForwardPlan f;
   Carve c;
-  f.nchunks = (int)((M + kDecodeMaxTokens - 1) / kDecodeMaxTokens);
+  f.variant = decode_variant(p->d_pad, p->nls, p->g, (int)std::min<int64_t>(M, kDecodeWideTokens));
+  f.chunk_tokens = decode_variant_tokens(f.variant);
+  f.nchunks = (int)((M + f.chunk_tokens - 1) / f.chunk_tokens);
   f.partial_off = c.take(prepass_partial_bytes((int)M, p->lr, p->d));
-  f.ts_off = c.take((size_t)f.nchunks * std::max(p->nls, 1) * 1024);
+  // rank-r fragments, in 16-token chunks
+  f.ts_off = c.take((size_t)((M + kDecodeMaxTokens - 1) / kDecodeMaxTokens) * std::max(p->nls, 1) * 1024);
   if (ce) {
-    f.ce_part_off = c.take((size_t)decode_num_units(p) * decode_parts_per_unit() * M * sizeof(float2));
+    f.ce_part_off = c.take((size_t)decode_num_units(p, f.variant) * decode_parts_per_unit() * M * sizeof(float2));
     f.tlogit_off = c.take((size_t)M * sizeof(float));
   }
   f.total = c.off;
@@ -166,12 +171,13 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   dp.argmax = greedy;
   dp.ce_part = ce_mode ? at<float2>(p->ws, f.ce_part_off) : nullptr;
   dp.ce_tlogit = ce_mode ? at<float>(p->ws, f.tlogit_off) : nullptr;
-  const int grid = std::min(decode_num_units(p), p->sm_count);
+  const int units = decode_num_units(p, f.variant);
+  const int grid = std::min(units, p->sm_count);
+  dp.variant = f.variant;
   for (int c = 0; c < f.nchunks; ++c) {
-    dp.m0 = c * kDecodeMaxTokens;
-    dp.M = (int)std::min<int64_t>(kDecodeMaxTokens, M - dp.m0);
-    dp.variant = decode_variant(p->d_pad, p->nls, p->g, dp.M);
-    dp.ts = pp.ts + (size_t)c * p->nls * 256;
+    dp.m0 = c * f.chunk_tokens;
+    dp.M = (int)std::min<int64_t>(f.chunk_tokens, M - dp.m0);
+    dp.ts = pp.ts + (size_t)(dp.m0 / kDecodeMaxTokens) * p->nls * 256;
     cudaEvent_t ev = nullptr;
     timer_begin(p, "decode", s, &ev);
     // The first chunk overlaps the pre-pass grid (programmatic dependent launch).
@@ -183,7 +189,7 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   if (ce_mode) {
     cudaEvent_t ev = nullptr;
     timer_begin(p, "ce_finalize", s, &ev);
-    const int parts = decode_num_units(p) * decode_parts_per_unit();
+    const int parts = units * decode_parts_per_unit();
     cudaError_t e =
         greedy   ? launch_argmax_finalize(dp.ce_part, parts, (int)M, amax_idx, amax_val, s)
         : parts3 ? launch_lse_partial_finalize(dp.ce_part, parts, dp.ce_tlogit, targets, row0, p->V, (int)M, parts3, s)
@@ -240,14 +246,20 @@ archead_status run_forward(archead_pack *p, const void *x, int64_t M, void *out,
   if (path != ARCHEAD_PATH_AUTO && path != ARCHEAD_PATH_DECODE && path != ARCHEAD_PATH_PREFILL)
     return ARCHEAD_ERR_INVALID_ARG;
   AH_CUDA(cudaSetDevice(p->device));
-  // AUTO: the decode kernel streams the head once per 16 tokens; a prefill
-  // launch computes full 256-token tiles and costs about four decode passes
-  // for M <= 256 (Qwen3-8B shape: ~360 us against ~95 us a pass), so up to
-  // three decode passes win.  Heads too wide for the decode kernel's shared
-  // memory plan (per-group sums of x for 16 tokens, e.g. d = 2^20 at g = 32)
-  // take the prefill kernel under AUTO.
-  const bool decode = path == ARCHEAD_PATH_DECODE ||
-                      (path == ARCHEAD_PATH_AUTO && M <= 3 * kDecodeMaxTokens && decode_supported(p->d_pad, p->nls, p->g));
+  // AUTO: one decode launch streams the head once for up to 64 tokens (16,
+  // 32 or 64 per instance); a prefill launch computes full 256-token tiles
+  // and costs about as much as one 64-token decode launch plus a fifth
+  // (Qwen3-8B shape: ~350 us against ~150 us at 32 tokens and ~280 us at 64),
+  // so AUTO decodes up to 64 tokens when that takes at most three launches
+  // (heads too wide for the wide instances' ring run 16-token chunks).
+  // Heads too wide for the decode kernel's shared memory plan (per-group
+  // sums of x for 16 tokens, e.g. d = 2^20 at g = 32) take the prefill
+  // kernel under AUTO.
+  bool decode = path == ARCHEAD_PATH_DECODE;
+  if (path == ARCHEAD_PATH_AUTO && M <= kDecodeWideTokens && decode_supported(p->d_pad, p->nls, p->g)) {
+    const int tok = decode_variant_tokens(decode_variant(p->d_pad, p->nls, p->g, (int)M));
+    decode = (M + tok - 1) / tok <= 3;
+  }
   if (decode) return run_decode(p, x, M, out, out_fp32, targets, ce, amax_idx, amax_val, row0, parts3, s);
   return run_prefill(p, x, M, out, out_fp32, targets, ce, amax_idx, amax_val, row0, parts3, s);
 }

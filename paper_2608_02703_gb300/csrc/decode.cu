@@ -1,10 +1,16 @@
 // Host entry points of the decode kernel (decode_kernel.cuh); the INT8
 // format's instances compile here, the SC4 format's in decode_sc4.cu.
+#include <algorithm>
+
 #include "decode_kernel.cuh"
 
 namespace archead {
 
-int decode_num_units(const archead_pack *p) { return (p->num_tiles + kDecTiles - 1) / kDecTiles; }
+int decode_num_units(const archead_pack *p, int variant) {
+  return (p->num_tiles + variant_tiles(variant) - 1) / variant_tiles(variant);
+}
+
+int decode_variant_tokens(int variant) { return variant_tokens(variant); }
 
 int decode_parts_per_unit() { return kDecWarps; }
 
@@ -16,7 +22,17 @@ bool decode_supported(int d_pad, int nls, int g) {
 // of at least 96 KB; otherwise, and for 9..16 tokens, the instance that
 // streams x through the ring (very wide heads: 8 tokens of d = 16384 would
 // take 256 KB).
+// 17..32 and 33..64 tokens take the wide instances (one launch streams the
+// head once for all of them) while their ring keeps at least four stages,
+// else 16-token chunks of kDecStreamed2.  More than 64 tokens run in chunks
+// of 64 (kDecWide8 for every chunk, the last one included).
+static bool wide_fits(int d_pad, int nls, int g, int variant) {
+  return decode_plan(d_pad, nls, g, variant_tokens(variant), variant).stages >= 4;
+}
+
 int decode_variant(int d_pad, int nls, int g, int M) {
+  if (M > 32 && wide_fits(d_pad, nls, g, kDecWide8)) return kDecWide8;
+  if (M > 16 && wide_fits(d_pad, nls, g, kDecWide4)) return kDecWide4;
   if (M > 8) return kDecStreamed2;
   const DecodePlan pl = decode_plan(d_pad, nls, g, M, kDecResident1);
   return pl.stages >= 2 && pl.xs_off >= (size_t)96 * 1024 ? kDecResident1 : kDecStreamed2;
@@ -33,10 +49,10 @@ cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool
 // each variant needs the most shared memory.
 cudaError_t prepare_decode(const archead_pack *p) {
   if (!decode_supported(p->d_pad, p->nls, p->g)) return cudaSuccess;
-  DecodeParams dp = decode_params(p, nullptr, kDecodeMaxTokens);
-  for (int M : {8, kDecodeMaxTokens}) {
-    dp.M = M;
+  DecodeParams dp = decode_params(p, nullptr, kDecodeWideTokens);
+  for (int M : {8, 16, 32, kDecodeWideTokens}) {
     dp.variant = decode_variant(p->d_pad, p->nls, p->g, M);
+    dp.M = std::min(M, variant_tokens(dp.variant));
     const cudaError_t e = launch_decode(dp, 0, nullptr, false);
     if (e != cudaSuccess) return e;
   }

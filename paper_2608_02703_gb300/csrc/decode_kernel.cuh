@@ -34,8 +34,6 @@ namespace archead {
 
 constexpr int kDecWarps = 8;                      // consumer warps
 constexpr int kDecThreads = (kDecWarps + 1) * 32; // + producer warp
-constexpr int kDecTiles = 4;                      // 128-row tiles per unit
-constexpr int kDecMT = 4;                         // m-tiles per consumer warp (2 warps per tile)
 constexpr int kSmemLimit = 227 * 1024;
 
 // Kernel instances ("variants"), chosen per launch from the token count and
@@ -55,24 +53,42 @@ constexpr int kSmemLimit = 227 * 1024;
 // kept): 16 tokens of x resident as fp16 with a 2-chunk ring (98.4 us at
 // M = 16 against 94.8) or a 1-chunk ring with the next stage prefetched into
 // registers (114 us); 1-chunk stages for M <= 8 (98 us at M = 1 against 65).
-enum DecodeVariant { kDecResident1 = 0, kDecStreamed2 = 1 };
+//  - kDecWide4, kDecWide8: 17..32 and 33..64 tokens (four and eight n-tiles)
+//    with x streamed as above.  A warp owns 2 m-tiles (4 warps per tile,
+//    units of two tiles) resp. 1 m-tile (8 warps per tile, units of one
+//    tile), so that one unpacked code word feeds 8 MMAs in either and the
+//    head is streamed once per 32 resp. 64 tokens.
+enum DecodeVariant { kDecResident1 = 0, kDecStreamed2 = 1, kDecWide4 = 2, kDecWide8 = 3 };
 
-__host__ __device__ constexpr int variant_nt(int v) { return v == kDecResident1 ? 1 : 2; }
-__host__ __device__ constexpr bool streams_x(int v) { return v == kDecStreamed2; }
+__host__ __device__ constexpr int variant_nt(int v) {  // 8-token n-tiles
+  return v == kDecResident1 ? 1 : v == kDecStreamed2 ? 2 : v == kDecWide4 ? 4 : 8;
+}
+__host__ __device__ constexpr int variant_mt(int v) {  // 16-row m-tiles per consumer warp
+  return v == kDecWide4 ? 2 : v == kDecWide8 ? 1 : 4;
+}
+__host__ __device__ constexpr int variant_tiles(int v) { return variant_mt(v); }  // 8 warps x MT m-tiles / 8 per tile
+__host__ __device__ constexpr int variant_tokens(int v) { return 8 * variant_nt(v); }  // largest M of one launch
+__host__ __device__ constexpr bool streams_x(int v) { return v != kDecResident1; }
+// Token stride of the per-group sums of x (at least 16: the smallest instances' layout).
+__host__ __device__ constexpr int xsum_tokens(int v) { return variant_tokens(v) < 16 ? 16 : variant_tokens(v); }
 // 64-wide chunks of d per ring stage.  The shared-memory plan and the kernel
 // instance launched both take it from here.
 __host__ __device__ constexpr int stage_chunks(int v) { return 2; }
-constexpr int kXChunkBytes = 16 * kChunkK * 2;  // 16 tokens x 64 of d, bf16, 128-byte swizzle
+// One chunk of x in a stage: the instance's tokens x 64 of d, bf16, 128-byte swizzle.
+__host__ __device__ constexpr int x_chunk_bytes(int v) { return variant_tokens(v) < 16 ? 16 * kChunkK * 2 : variant_tokens(v) * kChunkK * 2; }
 
-// Stage geometry for SC chunks (64 of d each) per stage.
-template <int SC, bool XS>
+// Stage geometry for SC chunks (64 of d each) per stage, TL tiles per unit
+// and XB bytes of x per chunk (0: x not streamed).
+template <int SC, int TL, int XB>
 struct StageGeom {
-  static constexpr int kCodeBytes = kDecTiles * SC * kChunkBytes;  // also holds 2*SC low-rank steps per tile
+  static constexpr int kCodeBytes = TL * SC * kChunkBytes;  // also holds 2*SC low-rank steps per tile
   static constexpr int kScaleBytesPerTile = (SC * kChunkK / 32) * kTileRows * 2;  // up to SC*64/g groups (g >= 32)
-  static constexpr int kXOff = kCodeBytes + kDecTiles * kScaleBytesPerTile;       // a multiple of 1024
-  static constexpr int kBytes = kXOff + (XS ? SC * kXChunkBytes : 0);
+  static constexpr int kXOff = (kCodeBytes + TL * kScaleBytesPerTile + 1023) / 1024 * 1024;  // 1 KB aligned
+  static constexpr int kBytes = kXOff + SC * XB;
   static constexpr int kLrSteps = 2 * SC;  // 16-wide low-rank steps per stage (2 KB per tile each)
 };
+template <int V>
+using GeomOf = StageGeom<stage_chunks(V), variant_tiles(V), streams_x(V) ? x_chunk_bytes(V) : 0>;
 
 struct DecodePlan {
   int stages, sc;
@@ -89,11 +105,14 @@ static DecodePlan decode_plan(int d_pad, int nls, int g, int M, int variant) {
   DecodePlan pl{};
   const bool xs = streams_x(variant);
   pl.sc = stage_chunks(variant);
-  const size_t stage_bytes = pl.sc == 2 ? (xs ? StageGeom<2, true>::kBytes : StageGeom<2, false>::kBytes)
-                                        : (xs ? StageGeom<1, true>::kBytes : StageGeom<1, false>::kBytes);
+  const size_t stage_bytes = variant == kDecResident1   ? GeomOf<kDecResident1>::kBytes
+                             : variant == kDecStreamed2 ? GeomOf<kDecStreamed2>::kBytes
+                             : variant == kDecWide4     ? GeomOf<kDecWide4>::kBytes
+                                                        : GeomOf<kDecWide8>::kBytes;
   const size_t xs_bytes = xs ? 0 : (size_t)M * xs_row_elems(d_pad) * 2;
-  const size_t ts_bytes = (size_t)nls * 1024;
-  const size_t xsum_bytes = ((size_t)2 * (d_pad / g) * kDecodeMaxTokens + kDecodeMaxTokens) * 4;
+  // rank-r fragments of the 16-token chunks the launch covers
+  const size_t ts_bytes = (size_t)((variant_tokens(variant) + kDecodeMaxTokens - 1) / kDecodeMaxTokens) * nls * 1024;
+  const size_t xsum_bytes = ((size_t)2 * (d_pad / g) * xsum_tokens(variant) + xsum_tokens(variant)) * 4;
   const size_t fixed = xs_bytes + ts_bytes + xsum_bytes + 256;
   const size_t shared_cap = (size_t)kSmemLimit - prepass_smem(M) - 2048;
   int st = 8;
@@ -156,7 +175,11 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
   constexpr int NT = variant_nt(VAR);
   constexpr bool kStreamX = streams_x(VAR);
   constexpr bool kF16 = !kStreamX;  // fp16 operands with x staged in shared memory
-  using Geom = StageGeom<SC, kStreamX>;
+  constexpr int MT = variant_mt(VAR);        // m-tiles per consumer warp
+  constexpr int TL = variant_tiles(VAR);     // 128-row tiles per unit
+  constexpr int XT = xsum_tokens(VAR);       // token stride of the per-group sums
+  constexpr int XCB = x_chunk_bytes(VAR);    // one chunk of streamed x
+  using Geom = GeomOf<VAR>;
   constexpr int SS = 4 * SC;  // 16-wide k steps per stage
   // The kernel has no static shared memory, so the dynamic window starts on a
   // 1 KB boundary, which the 128-byte-swizzled x boxes rely on (checked
@@ -183,7 +206,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
   const int KC = p.d_pad / kChunkK;
   const int res_stages = KC / SC;
   const int lr_stages = (p.nls + Geom::kLrSteps - 1) / Geom::kLrSteps;
-  const int num_units = (p.num_tiles + kDecTiles - 1) / kDecTiles;
+  const int num_units = (p.num_tiles + TL - 1) / TL;
   const int xrow = xs_row_elems(p.d_pad);
 
   // Columns [d, d_pad) of the hidden states meet zero codes; zero them so
@@ -224,15 +247,16 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
     bool t_loaded = false;
     int it = 0;
     for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x) {
-      const int ntile = min(kDecTiles, p.num_tiles - kDecTiles * unit);
+      const int ntile = min(TL, p.num_tiles - TL * unit);
       for (int s = 0; s < res_stages + lr_stages; ++s, ++it) {
         const int st = it % stages;
         if (s == res_stages && !t_loaded) {
           // The rank-r fragments come from the pre-pass grid.
           asm volatile("griddepcontrol.wait;\n" ::: "memory");
-          if (leader) {
-            mbar_arrive_expect_tx(tbar, (uint32_t)(p.nls * 1024));
-            bulk_g2s(smem + ts_off, p.ts, (uint32_t)(p.nls * 1024), tbar);
+          if (leader) {  // the t fragments of the 16-token chunks this launch holds
+            const uint32_t tb = (uint32_t)(((p.M + kDecodeMaxTokens - 1) / kDecodeMaxTokens) * p.nls * 1024);
+            mbar_arrive_expect_tx(tbar, tb);
+            bulk_g2s(smem + ts_off, p.ts, tb, tbar);
           }
           t_loaded = true;
         }
@@ -249,13 +273,13 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
           const int nbr = (g1 >> 1) - (g0 >> 1) + 1;
           const int sbytes = kSC4 ? nbr * kTileRows : ng * kTileRows * 2;
           mbar_arrive_expect_tx(&full[st],
-                                (uint32_t)(ntile * (SC * kChunkBytes + sbytes) + (kStreamX ? SC * kXChunkBytes : 0)));
+                                (uint32_t)(ntile * (SC * kChunkBytes + sbytes) + (kStreamX ? SC * XCB : 0)));
           if (kStreamX) {
             for (int c = 0; c < SC; ++c)
-              tma_load_2d(buf + Geom::kXOff + c * kXChunkBytes, &p.tmap_x, (kc0 + c) * kChunkK, p.m0, &full[st]);
+              tma_load_2d(buf + Geom::kXOff + c * XCB, &p.tmap_x, (kc0 + c) * kChunkK, p.m0, &full[st]);
           }
           for (int t = 0; t < ntile; ++t) {
-            const int64_t vt = (int64_t)kDecTiles * unit + t;
+            const int64_t vt = (int64_t)TL * unit + t;
             bulk_g2s_hint(buf + t * SC * kChunkBytes, p.codes + (vt * KC + kc0) * kChunkBytes, SC * kChunkBytes,
                           &full[st], stream_policy);
             if constexpr (kSC4)
@@ -273,7 +297,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
           mbar_arrive_expect_tx(&full[st], (uint32_t)(ntile * (nl * kLrStepBytes + (last ? kTileRows * 2 : 0) +
                                                                 (first_sc4 ? kTileRows * 2 : 0))));
           for (int t = 0; t < ntile; ++t) {
-            const int64_t vt = (int64_t)kDecTiles * unit + t;
+            const int64_t vt = (int64_t)TL * unit + t;
             bulk_g2s_hint(buf + t * Geom::kLrSteps * kLrStepBytes, p.lr_codes + (vt * p.nls + ls0) * kLrStepBytes,
                           nl * kLrStepBytes, &full[st], stream_policy);
             if (last)
@@ -300,16 +324,16 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
   }
 
   // ---------------- consumer warps ----------------
-  const int tsel = warp / (8 / kDecMT);              // tile of the unit
-  const int mi0 = (warp % (8 / kDecMT)) * kDecMT;    // first of the warp's m-tiles in that tile
+  const int tsel = warp / (8 / MT);              // tile of the unit
+  const int mi0 = (warp % (8 / MT)) * MT;    // first of the warp's m-tiles in that tile
   const int gq = lane >> 2, cq = lane & 3;
   const int ng = p.d_pad / p.g;
-  float *tscale = xsum_s + 2 * ng * kDecodeMaxTokens;
+  float *tscale = xsum_s + 2 * ng * XT;
   if (kStreamX) {
     // Per-group sums of x for removing the bf16 operand bias (136), read
     // straight from global memory; no staging scale.
-    for (int e = threadIdx.x; e < ng * kDecodeMaxTokens; e += kDecWarps * 32) {
-      const int grp = e / kDecodeMaxTokens, m = e % kDecodeMaxTokens;
+    for (int e = threadIdx.x; e < ng * XT; e += kDecWarps * 32) {
+      const int grp = e / XT, m = e % XT;
       float sum = 0.f;
       if (m < p.M && grp * p.g < p.d) {
         const uint4 *src = reinterpret_cast<const uint4 *>(p.x + (int64_t)(p.m0 + m) * p.d + (int64_t)grp * p.g);
@@ -320,9 +344,9 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
         }
       }
       xsum_s[e] = -kInt4Bias * sum;
-      xsum_s[ng * kDecodeMaxTokens + e] = -kInt4Bias * sum;
+      xsum_s[ng * XT + e] = -kInt4Bias * sum;
     }
-    if (threadIdx.x < kDecodeMaxTokens) tscale[threadIdx.x] = 1.f;
+    if (threadIdx.x < XT) tscale[threadIdx.x] = 1.f;
     asm volatile("bar.sync 1, %0;\n" ::"r"(kDecWarps * 32) : "memory");  // consumer warps only
   } else {
     const bool ok = mbar_wait_warp(xbar, 0, p.wait_budget, abort_flag, p.err);
@@ -330,7 +354,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
       // Per-token power of two 2^-e that brings max |x| into [2^14, 2^15)
       // (fp16 range, and small tokens away from fp16 subnormals); tscale[m]
       // = 2^e undoes it after the residual.
-      for (int m = warp; m < kDecodeMaxTokens; m += kDecWarps) {
+      for (int m = warp; m < XT; m += kDecWarps) {
         uint32_t mx = 0;
         if (m < p.M) {
           const uint32_t *row = reinterpret_cast<const uint32_t *>(xs_s + m * xrow);
@@ -347,8 +371,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
       asm volatile("bar.sync 1, %0;\n" ::"r"(kDecWarps * 32) : "memory");
       // Convert each token's row to fp16 in place, group by group, and sum
       // the values the MMAs will see (for removing the operand bias).
-      for (int e = threadIdx.x; e < ng * kDecodeMaxTokens; e += kDecWarps * 32) {
-        const int grp = e / kDecodeMaxTokens, m = e % kDecodeMaxTokens;
+      for (int e = threadIdx.x; e < ng * XT; e += kDecWarps * 32) {
+        const int grp = e / XT, m = e % XT;
         float sum = 0.f;
         if (m < p.M) {
           const float inv = 1.f / tscale[m];  // exact: a power of two
@@ -362,7 +386,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
           }
         }
         xsum_s[e] = -kF16BiasLo * sum;
-        xsum_s[ng * kDecodeMaxTokens + e] = -kF16BiasHi * sum;
+        xsum_s[ng * XT + e] = -kF16BiasHi * sum;
       }
     }
     asm volatile("bar.sync 1, %0;\n" ::"r"(kDecWarps * 32) : "memory");  // consumer warps only
@@ -385,12 +409,12 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
   int st = 0;     // ring slot
   uint32_t ph = 0;  // its phase parity
   for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x) {
-    const int ntile = min(kDecTiles, p.num_tiles - kDecTiles * unit);
+    const int ntile = min(TL, p.num_tiles - TL * unit);
     const bool active = tsel < ntile;
-    float acc[kDecMT][NT][4];
-    float part[kDecMT][NT][4];  // one group's sums; each group's first MMA starts from zero
+    float acc[MT][NT][4];
+    float part[MT][NT][4];  // one group's sums; each group's first MMA starts from zero
 #pragma unroll
-    for (int a = 0; a < kDecMT; ++a)
+    for (int a = 0; a < MT; ++a)
 #pragma unroll
       for (int b = 0; b < NT; ++b)
 #pragma unroll
@@ -403,8 +427,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
     constexpr int NGS = GS <= SS ? SS / GS : 1;  // groups whose scales a stage carries
     for (int s = 0; s < res_stages; ++s) {
       if (!mbar_wait_warp(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
-      uint4 w[kStreamX ? 1 : SC][kDecMT];
-      float s_lo[NGS][kDecMT], s_hi[NGS][kDecMT];
+      uint4 w[kStreamX ? 1 : SC][MT];
+      float s_lo[NGS][MT], s_hi[NGS][MT];
       const uint8_t *sbuf = smem + (size_t)st * Geom::kBytes;
       const uint8_t *cb = sbuf + tsel * SC * kChunkBytes + mi0 * 512 + lane * 16;
       if (active) {
@@ -414,7 +438,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
 #pragma unroll
           for (int c = 0; c < (kStreamX ? 1 : SC); ++c)
 #pragma unroll
-            for (int mt = 0; mt < kDecMT; ++mt)
+            for (int mt = 0; mt < MT; ++mt)
               w[c][mt] = *reinterpret_cast<const uint4 *>(cb + c * kChunkBytes + mt * 512);
         }
         if constexpr (kSC4) {
@@ -426,7 +450,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
             const int ggl = gfirst + gi;
             const int br = (ggl >> 1) - (gfirst >> 1), sh = 4 * (ggl & 1);
 #pragma unroll
-            for (int mt = 0; mt < kDecMT; ++mt) {
+            for (int mt = 0; mt < MT; ++mt) {
               s_lo[gi][mt] = scale_mult(sc8[br * kTileRows + mt * 16], sh);
               const uint32_t bh = sc8[br * kTileRows + mt * 16 + 8];
               s_hi[gi][mt] = kF16 ? scale_mult_16th(bh, sh) : scale_mult(bh, sh);  // fp16 operands: x16 rows
@@ -436,7 +460,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
 #pragma unroll
           for (int gi = 0; gi < NGS; ++gi)
 #pragma unroll
-            for (int mt = 0; mt < kDecMT; ++mt) {
+            for (int mt = 0; mt < MT; ++mt) {
               s_lo[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16]);
               s_hi[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16 + 8]) * (kF16 ? 0.0625f : 1.f);  // fp16: x16
             }
@@ -454,21 +478,25 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
       for (int c = 0; c < SC; ++c) {
         if (kStreamX) {
 #pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt)
+          for (int mt = 0; mt < MT; ++mt)
             w[0][mt] = *reinterpret_cast<const uint4 *>(cb + c * kChunkBytes + mt * 512);
         }
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           const int ks = c * 4 + j;  // k step within the stage
           uint32_t b[NT][2];
-          if constexpr (kStreamX && NT == 2) {
-            // Matrices (tokens 0-7 | 8-15) x (k 0-7 | 8-15) of the k step: lane
-            // L addresses token 8 (L / 16) + L % 8 at 16-byte chunk 2j + (L / 8) % 2
-            // of its 128-byte row (chunk index XOR token % 8).
-            const int tok = 8 * (lane >> 4) + (lane & 7);
-            ldsm_x4(smem_u32(sbuf + Geom::kXOff + c * kXChunkBytes + tok * 128 +
-                             (((2 * j + ((lane >> 3) & 1)) ^ (tok & 7)) << 4)),
-                    b[0][0], b[0][1], b[1][0], b[1][1]);
+          if constexpr (kStreamX && NT >= 2) {
+            // Per 16 tokens q: matrices (tokens 16q + 0-7 | 8-15) x (k 0-7 |
+            // 8-15) of the k step: lane L addresses token 16q + 8 (L / 16) +
+            // L % 8 at 16-byte chunk 2j + (L / 8) % 2 of its 128-byte row
+            // (chunk index XOR token % 8).
+#pragma unroll
+            for (int q = 0; q < NT / 2; ++q) {
+              const int tok = 16 * q + 8 * (lane >> 4) + (lane & 7);
+              ldsm_x4(smem_u32(sbuf + Geom::kXOff + c * XCB + tok * 128 +
+                               (((2 * j + ((lane >> 3) & 1)) ^ (tok & 7)) << 4)),
+                      b[2 * q][0], b[2 * q][1], b[2 * q + 1][0], b[2 * q + 1][1]);
+            }
           } else if constexpr (!kStreamX && NT == 1 && kSC4) {
             // Tokens 0-7 (clamped to M) x (k 0-7 | 8-15) of the k step.  (The
             // INT8 format's resident instance keeps its two 32-bit loads: its
@@ -479,7 +507,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
               if (kStreamX) {
-                const uint8_t *xr = sbuf + Geom::kXOff + c * kXChunkBytes + (8 * nt + gq) * 128 + 4 * cq;
+                const uint8_t *xr = sbuf + Geom::kXOff + c * XCB + (8 * nt + gq) * 128 + 4 * cq;
                 b[nt][0] = *reinterpret_cast<const uint32_t *>(xr + (((2 * j) ^ gq) << 4));
                 b[nt][1] = *reinterpret_cast<const uint32_t *>(xr + (((2 * j + 1) ^ gq) << 4));
               } else {
@@ -500,13 +528,14 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
             const int ggl = GS <= SS ? s * (SS / GS) + ks / GS : s / (GS / SS);  // group index along d
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
-              const int o = ggl * kDecodeMaxTokens + 8 * nt + 2 * cq;
+              const int o = ggl * XT + 8 * nt + 2 * cq;
               nb_lo[nt] = *reinterpret_cast<const float2 *>(xsum_s + o);
-              nb_hi[nt] = *reinterpret_cast<const float2 *>(xsum_s + ng * kDecodeMaxTokens + o);
+              // bf16 operands carry one bias (136) on both row halves
+              nb_hi[nt] = kStreamX ? nb_lo[nt] : *reinterpret_cast<const float2 *>(xsum_s + ng * XT + o);
             }
           }
 #pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt) {
+          for (int mt = 0; mt < MT; ++mt) {
             const uint4 wv = w[kStreamX ? 0 : c][mt];
             const uint32_t word = j == 0 ? wv.x : j == 1 ? wv.y : j == 2 ? wv.z : wv.w;
             uint32_t a[4];
@@ -535,7 +564,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
           if (boundary) {
             const int gi = GS <= SS ? ks / GS : 0;  // group within the stage
 #pragma unroll
-            for (int mt = 0; mt < kDecMT; ++mt) promote<NT>(acc[mt], part[mt], s_lo[gi][mt], s_hi[gi][mt]);
+            for (int mt = 0; mt < MT; ++mt) promote<NT>(acc[mt], part[mt], s_lo[gi][mt], s_hi[gi][mt]);
           }
         }
       }
@@ -547,7 +576,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
 
     // Back to the hidden states' own scale (exact: powers of two).
 #pragma unroll
-    for (int a = 0; a < (kF16 ? kDecMT : 0); ++a)
+    for (int a = 0; a < (kF16 ? MT : 0); ++a)
 #pragma unroll
       for (int b = 0; b < NT; ++b) {
         acc[a][b][0] *= unscale[b].x;
@@ -557,9 +586,9 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
       }
     // SC4 without rank-r branches: no stage carries the row scales; read them here.
     if (kSC4 && lr_stages == 0 && active) {
-      const int64_t rb = ((int64_t)kDecTiles * unit + tsel) * kTileRows + mi0 * 16 + gq;
+      const int64_t rb = ((int64_t)TL * unit + tsel) * kTileRows + mi0 * 16 + gq;
 #pragma unroll
-      for (int mt = 0; mt < kDecMT; ++mt) {
+      for (int mt = 0; mt < MT; ++mt) {
         const float r_lo = fp16_bits_to_f32(p.s_row[rb + mt * 16]), r_hi = fp16_bits_to_f32(p.s_row[rb + mt * 16 + 8]);
 #pragma unroll
         for (int b = 0; b < NT; ++b) {
@@ -574,7 +603,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
     // Rank-r branches as extra k steps (core: factor 1; correction: row scale
     // of A_w), with the same copy-then-release of each stage.
 #pragma unroll
-    for (int a = 0; a < kDecMT; ++a)
+    for (int a = 0; a < MT; ++a)
 #pragma unroll
       for (int b = 0; b < NT; ++b)
 #pragma unroll
@@ -588,20 +617,20 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
       const int ls0 = s * Geom::kLrSteps;
       const int nl = min(Geom::kLrSteps, p.nls - ls0);
       const bool last_stage = s == lr_stages - 1;
-      uint2 lw[Geom::kLrSteps][kDecMT];
-      float a_lo[kDecMT], a_hi[kDecMT];
+      uint2 lw[Geom::kLrSteps][MT];
+      float a_lo[MT], a_hi[MT];
       if (active) {
         const uint8_t *buf = smem + (size_t)st * Geom::kBytes;
 #pragma unroll
         for (int l = 0; l < Geom::kLrSteps; ++l)
 #pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt)
+          for (int mt = 0; mt < MT; ++mt)
             if (l < nl)
               lw[l][mt] = *reinterpret_cast<const uint2 *>(
                   buf + ((size_t)(tsel * Geom::kLrSteps + l) * 8 + mi0 + mt) * 256 + lane * 8);
         const uint16_t *sa = reinterpret_cast<const uint16_t *>(buf + Geom::kCodeBytes + tsel * Geom::kScaleBytesPerTile);
 #pragma unroll
-        for (int mt = 0; mt < kDecMT; ++mt) {
+        for (int mt = 0; mt < MT; ++mt) {
           const int r = (mi0 + mt) * 16 + gq;
           a_lo[mt] = last_stage ? fp16_bits_to_f32(sa[r]) : 0.f;
           a_hi[mt] = last_stage ? fp16_bits_to_f32(sa[r + 8]) : 0.f;
@@ -609,7 +638,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
         if (kSC4 && s == 0) {
           // The residual's row scales (SC4), before any rank-r term is added.
 #pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt) {
+          for (int mt = 0; mt < MT; ++mt) {
             const int r = (mi0 + mt) * 16 + gq;
             const float r_lo = fp16_bits_to_f32(sa[kTileRows + r]), r_hi = fp16_bits_to_f32(sa[kTileRows + r + 8]);
 #pragma unroll
@@ -633,15 +662,17 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
         uint32_t bh[NT][2], bl[NT][2];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
-          const uint2 h2 = *reinterpret_cast<const uint2 *>(ts_s + ((((size_t)ls * 2 + 0) * 2 + nt) * 32 + lane) * 2);
-          const uint2 l2 = *reinterpret_cast<const uint2 *>(ts_s + ((((size_t)ls * 2 + 1) * 2 + nt) * 32 + lane) * 2);
+          // t fragments of the 16-token chunk holding n-tile nt
+          const uint32_t *tc = ts_s + (size_t)(nt >> 1) * p.nls * 256;
+          const uint2 h2 = *reinterpret_cast<const uint2 *>(tc + ((((size_t)ls * 2 + 0) * 2 + (nt & 1)) * 32 + lane) * 2);
+          const uint2 l2 = *reinterpret_cast<const uint2 *>(tc + ((((size_t)ls * 2 + 1) * 2 + (nt & 1)) * 32 + lane) * 2);
           bh[nt][0] = h2.x;
           bh[nt][1] = h2.y;
           bl[nt][0] = l2.x;
           bl[nt][1] = l2.y;
         }
 #pragma unroll
-        for (int mt = 0; mt < kDecMT; ++mt) {
+        for (int mt = 0; mt < MT; ++mt) {
           uint32_t a[4];
           unpack_int8x8(lw[l][mt].x, lw[l][mt].y, a);
 #pragma unroll
@@ -653,7 +684,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
         if (ls + 1 == p.nls_core || ls + 1 == p.nls) {
           const bool corr = ls + 1 == p.nls && p.nls > p.nls_core;  // the correction ends with the last stage
 #pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt) {
+          for (int mt = 0; mt < MT; ++mt) {
             promote<NT>(acc[mt], part[mt], corr ? a_lo[mt] : 1.f, corr ? a_hi[mt] : 1.f);
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt)
@@ -665,11 +696,11 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
     }
 
     // Epilogue.  acc[mt][nt][i]: row 16*(mi0+mt) + gq + 8*(i/2), token 8*nt + 2*cq + i%2.
-    const int64_t row_base = ((int64_t)kDecTiles * unit + tsel) * kTileRows;
+    const int64_t row_base = ((int64_t)TL * unit + tsel) * kTileRows;
     if (p.out) {
       if (active) {
 #pragma unroll
-        for (int mt = 0; mt < kDecMT; ++mt)
+        for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
@@ -696,7 +727,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
           float bv = -INFINITY;
           int bi = 0x7fffffff;
 #pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt)
+          for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
             for (int ih = 0; ih < 2; ++ih) {
               const int64_t row = row_base + (mi0 + mt) * 16 + gq + 8 * ih;
@@ -726,10 +757,10 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
         for (int tl = 0; tl < 2; ++tl) {
           const int tok = nt * 8 + 2 * cq + tl;
           const int tgt = tok < p.M ? p.targets[p.m0 + tok] - p.row0 : -1;  // this pack's row numbering
-          float vals[2 * kDecMT];
+          float vals[2 * MT];
           float mx = -INFINITY;
 #pragma unroll
-          for (int mt = 0; mt < kDecMT; ++mt)
+          for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
             for (int ih = 0; ih < 2; ++ih) {
               const int64_t row = row_base + (mi0 + mt) * 16 + gq + 8 * ih;
@@ -741,7 +772,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
             }
           float sum = 0.f;
 #pragma unroll
-          for (int q = 0; q < 2 * kDecMT; ++q) sum += (vals[q] == -INFINITY) ? 0.f : __expf(vals[q] - mx);
+          for (int q = 0; q < 2 * MT; ++q) sum += (vals[q] == -INFINITY) ? 0.f : __expf(vals[q] - mx);
           LsePair lp{mx, sum};
 #pragma unroll
           for (int off = 4; off < 32; off <<= 1) {
@@ -793,12 +824,15 @@ template <bool kSC4>
 cudaError_t launch_decode_fmt(const DecodeParams &dp, int grid, cudaStream_t s, bool pdl) {
   const DecodePlan pl = decode_plan(dp.d_pad, dp.nls, dp.g, dp.M, dp.variant);
   if (pl.stages < 2 || pl.sc != stage_chunks(dp.variant)) return cudaErrorInvalidValue;
-  if (dp.M < 1 || dp.M > (variant_nt(dp.variant) == 1 ? 8 : 16)) return cudaErrorInvalidValue;
+  if (dp.M < 1 || dp.M > variant_tokens(dp.variant)) return cudaErrorInvalidValue;
   if (dp.variant == kDecResident1) return launch_g<kDecResident1, kSC4>(dp, grid, s, pl, pdl);
-  if (dp.variant != kDecStreamed2) return cudaErrorInvalidValue;
+  if (dp.variant < kDecStreamed2 || dp.variant > kDecWide8) return cudaErrorInvalidValue;
   DecodeParams dx = dp;
-  if (grid > 0 && !make_tma_map_bf16(&dx.tmap_x, dp.x, dp.M_total, dp.d, 16)) return cudaErrorInvalidValue;
-  return launch_g<kDecStreamed2, kSC4>(dx, grid, s, pl, pdl);
+  if (grid > 0 && !make_tma_map_bf16(&dx.tmap_x, dp.x, dp.M_total, dp.d, variant_tokens(dp.variant)))
+    return cudaErrorInvalidValue;
+  if (dp.variant == kDecStreamed2) return launch_g<kDecStreamed2, kSC4>(dx, grid, s, pl, pdl);
+  if (dp.variant == kDecWide4) return launch_g<kDecWide4, kSC4>(dx, grid, s, pl, pdl);
+  return launch_g<kDecWide8, kSC4>(dx, grid, s, pl, pdl);
 }
 
 

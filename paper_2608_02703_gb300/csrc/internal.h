@@ -49,12 +49,13 @@ constexpr int kTileRows = 128;     // vocabulary rows per tile
 constexpr int kChunkK = 64;        // d per code chunk
 constexpr int kChunkBytes = 4096;  // 128 rows x 64 codes / 2
 constexpr int kLrStepBytes = 2048; // 128 rows x 16 codes
-constexpr int kDecodeMaxTokens = 16;
+constexpr int kDecodeMaxTokens = 16;   // tokens per chunk of the rank-r fragments (and of noalloc calls)
+constexpr int kDecodeWideTokens = 64;  // tokens of the widest decode launch
 constexpr int kPrepassKSplit = 256;  // d per pre-pass block
 constexpr int64_t kDefaultWaitBudget = 2000000000LL;  // cycles, about one second
 
 struct DecodeParams {
-  CUtensorMap tmap_x;   // x [M_total][d] bf16, box 64 x 16 rows (kernel instances that stream x; M > 8)
+  CUtensorMap tmap_x;   // x [M_total][d] bf16, box 64 x (the instance's tokens) rows (instances that stream x)
   const uint8_t *codes;
   const uint16_t *scales;   // fp16 group scales (INT8 format)
   const uint8_t *scodes;    // 4-bit group-scale codes (SC4 format)
@@ -163,18 +164,20 @@ size_t prepass_partial_bytes(int M, int lr, int d);
 // pdl: launch as a programmatic dependent of the immediately preceding pre-pass grid.
 cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool pdl);
 // Shared-memory opt-in (and so module loading) of every decode kernel
-// instance this pack can launch for 1..16 tokens, done ahead of any launch.
+// instance this pack can launch, done ahead of any launch.
 cudaError_t prepare_decode(const archead_pack *p);
 // Tensor map of a bf16 [rows][cols] row-major matrix: box 64 columns x
 // box_rows rows, 128-byte swizzle, zero fill out of bounds.  False if the
 // driver entry point is missing or the encoder rejects the layout (base or
 // row pitch not 16-byte aligned).
 bool make_tma_map_bf16(CUtensorMap *map, const void *base, int64_t rows, int64_t cols, int box_rows);
-int decode_num_units(const archead_pack *p);
+int decode_num_units(const archead_pack *p, int variant);  // units (and ce partial blocks) of a variant
+int decode_variant_tokens(int variant);                    // tokens one launch of a variant takes
 int decode_parts_per_unit();
 bool decode_supported(int d_pad, int nls, int g);
-// Kernel instance to launch for M <= 16 tokens (0: one 8-token tile, x
-// resident; 1: two tiles, x resident; 2: two tiles, x streamed).
+// Kernel instance for a launch of M tokens (M > 64: the instance every
+// 64-token chunk runs): 0 one 8-token n-tile, x resident; 1, 2, 3 two, four
+// and eight n-tiles, x streamed.
 int decode_variant(int d_pad, int nls, int g, int M);
 cudaError_t launch_prefill(const archead_pack *pk, const void *x, int M, const uint16_t *T, void *out, int out_fp32,
                            bool argmax, const int32_t *targets, int row0, float2 *ce_part, float *ce_tlogit,

@@ -101,7 +101,7 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
 
   // The counters are the only state that must start at zero.
   e = cudaMemsetAsync(counters, 0, (size_t)pairs * sizeof(int), s);
-  // Every decode instance this pack can use (one or two 8-token tiles) is
+  // Every decode instance this pack can use (the wide ones included) is
   // opted into its shared memory here, so that a first call at any M leaves
   // nothing for a later call at another M to set up (inside a capture, say).
   if (e == cudaSuccess) e = prepare_decode(pack);
@@ -120,7 +120,7 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
   dp.variant = decode_variant(pack->d_pad, pack->nls, pack->g, (int)M);
   dp.out = logits;
   dp.out_fp32 = out_dtype == ARCHEAD_OUT_FP32;
-  const int units = decode_num_units(pack);
+  const int units = decode_num_units(pack, dp.variant);
   if (e == cudaSuccess) e = launch_decode(dp, units < pack->sm_count ? units : pack->sm_count, s, pack->lr > 0);
   if (e != cudaSuccess) {
     set_last_error_message(cudaGetErrorString(e));

@@ -79,7 +79,7 @@ def test_dequant_bit_exact(name):
 
 
 @pytest.mark.parametrize("name", sorted(SHAPES))
-@pytest.mark.parametrize("M", [1, 3, 8, 9, 16])
+@pytest.mark.parametrize("M", [1, 3, 8, 9, 16, 32, 64])
 def test_decode_logits(name, M):
     pack, head = get(name)
     shape = SHAPES[name]
@@ -168,7 +168,7 @@ def test_wide_head(shape):
     try:
         x = make_hidden(shape.d, 64, seed=5)
         ref = oracle.logits(head, shape, x)
-        for M in (1, 5, 8, 16):
+        for M in (1, 5, 8, 16, 27, 64):
             got = gu.forward(pack, x[:M], archead.OUT_FP32, archead.PATH_DECODE)
             gu.check_logits(got, ref[:M], where=f"d={shape.d} decode M={M}")
         got = gu.forward(pack, x, archead.OUT_FP32, archead.PATH_PREFILL)
