@@ -125,7 +125,7 @@ ForwardPlan plan_decode(archead_pack *p, int64_t M, bool ce) {
   // rank-r fragments, in 16-token chunks
   f.ts_off = c.take((size_t)((M + kDecodeMaxTokens - 1) / kDecodeMaxTokens) * std::max(p->nls, 1) * 1024);
   if (ce) {
-    f.ce_part_off = c.take((size_t)decode_num_units(p, f.variant) * decode_parts_per_unit() * M * sizeof(float2));
+    f.ce_part_off = c.take((size_t)decode_num_units(p, f.variant) * decode_parts_per_unit(f.variant) * M * sizeof(float2));
     f.tlogit_off = c.take((size_t)M * sizeof(float));
   }
   f.total = c.off;
@@ -189,7 +189,7 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   if (ce_mode) {
     cudaEvent_t ev = nullptr;
     timer_begin(p, "ce_finalize", s, &ev);
-    const int parts = units * decode_parts_per_unit();
+    const int parts = units * decode_parts_per_unit(f.variant);
     cudaError_t e =
         greedy   ? launch_argmax_finalize(dp.ce_part, parts, (int)M, amax_idx, amax_val, s)
         : parts3 ? launch_lse_partial_finalize(dp.ce_part, parts, dp.ce_tlogit, targets, row0, p->V, (int)M, parts3, s)

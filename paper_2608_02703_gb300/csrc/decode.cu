@@ -12,7 +12,7 @@ int decode_num_units(const archead_pack *p, int variant) {
 
 int decode_variant_tokens(int variant) { return variant_tokens(variant); }
 
-int decode_parts_per_unit() { return kDecWarps; }
+int decode_parts_per_unit(int variant) { return variant_cw(variant); }
 
 bool decode_supported(int d_pad, int nls, int g) {
   return decode_plan(d_pad, nls, g, kDecodeMaxTokens, kDecStreamed2).stages >= 2;

@@ -1,30 +1,34 @@
-// Memory-bound decode kernel (M <= 16 tokens) of the packed LM-head forward
-// (paper, Section 3.2, Eq. 7; Appendix B: the core and correction paths are
-// evaluated separately and no dense head is formed).
+// Memory-bound decode kernel (up to 64 tokens per launch) of the packed
+// LM-head forward (paper, Section 3.2, Eq. 7; Appendix B: the core and
+// correction paths are evaluated separately and no dense head is formed).
 //
-// Persistent grid, one block per SM.  A unit of work is 512 vocabulary rows
-// (four 128-row tiles).  One producer warp streams each unit's INT4 codes,
-// group scales and low-rank codes with 1-D bulk TMA copies into a ring of
-// shared-memory stages (mbarrier full/empty pairs).  Eight consumer warps each
-// own four 16-row m-tiles.  The hidden states are staged once per block by
-// TMA and converted in place to fp16, each token scaled by a power of two that
-// keeps it in fp16 range (exact for bf16 inputs in the normal range).  Per
-// 16-wide k step a consumer turns one 32-bit word of offset-binary nibbles
-// into the four fp16 A-fragment registers of an m16n8k16 MMA (exact biased
-// integers, see unpack_int4x8_f16) and multiplies them with the hidden states
-// (B fragments, tokens on the 8-wide side), accumulating in fp32.  At the end
-// of every quantisation group the bias is removed and the partial sums are
-// promoted by that row's group scale in fp32.  The rank-r
+// Persistent grid, one block per SM.  A unit of work is one to four 128-row
+// vocabulary tiles (by kernel instance, below).  One producer warp streams
+// each unit's INT4 codes, group scales and low-rank codes with 1-D bulk TMA
+// copies into a ring of shared-memory stages (mbarrier full/empty pairs).
+// Consumer warps each own 16-row m-tiles of the unit and 8-token n-tiles.
+// For up to 8 tokens the hidden states are staged once per block by TMA and
+// converted in place to fp16, each token scaled by a power of two that keeps
+// it in fp16 range (exact for bf16 inputs in the normal range); wider
+// instances stream x through the ring as bf16.  Per 16-wide k step a
+// consumer turns one 32-bit word of offset-binary nibbles into the four
+// A-fragment registers of an m16n8k16 MMA (exact biased integers, see
+// unpack_int4x8_f16 / unpack_int4x8_biased) and multiplies them with the
+// hidden states (B fragments, tokens on the 8-wide side), accumulating in
+// fp32.  The accumulators run in units of the current quantisation group's
+// scale: at the start of each group they are multiplied by the ratio of the
+// previous group's scale to this one's and given the group's bias term, and
+// the last group's scale multiplies the finished residual once.  The rank-r
 // branches follow as extra k steps: int8 codes of A_c (core) or A_w
 // (correction) times the bf16 hi/lo split of t = x V from the pre-pass, the
-// correction promoted by the row scale of A_w.  The pre-pass runs as the
+// correction in units of the row scale of A_w.  The pre-pass runs as the
 // preceding grid; this kernel starts streaming under programmatic dependent
 // launch and waits for the pre-pass only before the first rank-r stage.
 //
 // In the paper's packed format (SC4) a group scale is s_row * (q + 1) with a
-// 4-bit code q: the group promotion multiplies by q + 1 (read from the
-// stage's code bytes) and the row scale s_row, which the first rank-r stage
-// carries, multiplies the finished residual once per row.
+// 4-bit code q: the group ratios come from q + 1 (read from the stage's code
+// bytes) and the row scale s_row, which the first rank-r stage carries,
+// multiplies the finished residual once per row.
 #pragma once
 
 #include "device.cuh"
@@ -32,8 +36,6 @@
 
 namespace archead {
 
-constexpr int kDecWarps = 8;                      // consumer warps
-constexpr int kDecThreads = (kDecWarps + 1) * 32; // + producer warp
 constexpr int kSmemLimit = 227 * 1024;
 
 // Kernel instances ("variants"), chosen per launch from the token count and
@@ -54,19 +56,30 @@ constexpr int kSmemLimit = 227 * 1024;
 // M = 16 against 94.8) or a 1-chunk ring with the next stage prefetched into
 // registers (114 us); 1-chunk stages for M <= 8 (98 us at M = 1 against 65).
 //  - kDecWide4, kDecWide8: 17..32 and 33..64 tokens (four and eight n-tiles)
-//    with x streamed as above.  A warp owns 2 m-tiles (4 warps per tile,
-//    units of two tiles) resp. 1 m-tile (8 warps per tile, units of one
-//    tile), so that one unpacked code word feeds 8 MMAs in either and the
-//    head is streamed once per 32 resp. 64 tokens.
+//    with x streamed as above; the head is streamed once per 32 resp. 64
+//    tokens, in units of two tiles.  kDecWide4 runs sixteen consumer warps of
+//    one m-tile each (registers for a group's part sums at 96 a thread).
+//    kDecWide8 runs eight warps of two m-tiles each, so that every B
+//    fragment read from shared memory feeds two MMAs: with one m-tile a warp
+//    the ldmatrix traffic held it at 277 us for 64 tokens on the
+//    Qwen3-8B-shaped head, against 247 us.  Its 64 accumulators leave no
+//    registers for part sums: it keeps them in units of the group scale.
+//    Measured and not kept: kDecWide4 with eight warps of four m-tiles in
+//    group-scale units (145-152 us for 17-32 tokens, no better; 207 us with
+//    the paper's format, which spilled), and kDecWide8 with sixteen warps of
+//    two m-tiles and four n-tiles each (265-278 us).
 enum DecodeVariant { kDecResident1 = 0, kDecStreamed2 = 1, kDecWide4 = 2, kDecWide8 = 3 };
 
 __host__ __device__ constexpr int variant_nt(int v) {  // 8-token n-tiles
   return v == kDecResident1 ? 1 : v == kDecStreamed2 ? 2 : v == kDecWide4 ? 4 : 8;
 }
+__host__ __device__ constexpr int variant_cw(int v) { return v == kDecWide4 ? 16 : 8; }  // consumer warps
 __host__ __device__ constexpr int variant_mt(int v) {  // 16-row m-tiles per consumer warp
-  return v == kDecWide4 ? 2 : v == kDecWide8 ? 1 : 4;
+  return v == kDecWide4 ? 1 : v == kDecWide8 ? 2 : 4;
 }
-__host__ __device__ constexpr int variant_tiles(int v) { return variant_mt(v); }  // 8 warps x MT m-tiles / 8 per tile
+// 128-row tiles per unit: the consumer warps cover them, MT m-tiles each.
+__host__ __device__ constexpr int variant_tiles(int v) { return variant_cw(v) * variant_mt(v) / 8; }
+__host__ __device__ constexpr int variant_threads(int v) { return (variant_cw(v) + 1) * 32; }  // + producer warp
 __host__ __device__ constexpr int variant_tokens(int v) { return 8 * variant_nt(v); }  // largest M of one launch
 __host__ __device__ constexpr bool streams_x(int v) { return v != kDecResident1; }
 // Token stride of the per-group sums of x (at least 16: the smallest instances' layout).
@@ -170,9 +183,10 @@ __device__ __forceinline__ float scale_mult_16th(uint32_t b, int sh) {
 // VAR: DecodeVariant (n-tiles of 8 tokens, resident or streamed x); SC:
 // 64-wide chunks per stage; GS: 16-wide k steps per group.
 template <int VAR, int SC, int GS, bool kSC4>
-__global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_constant__ DecodeParams p, int stages,
+__global__ void __launch_bounds__(variant_threads(VAR), 1) decode_kernel(const __grid_constant__ DecodeParams p, int stages,
                                                                 int xs_off, int ts_off, int xsum_off, int bar_off) {
-  constexpr int NT = variant_nt(VAR);
+  constexpr int kDecWarps = variant_cw(VAR);  // consumer warps
+  constexpr int NT = variant_nt(VAR);          // n-tiles per warp
   constexpr bool kStreamX = streams_x(VAR);
   constexpr bool kF16 = !kStreamX;  // fp16 operands with x staged in shared memory
   constexpr int MT = variant_mt(VAR);        // m-tiles per consumer warp
@@ -181,6 +195,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
   constexpr int XCB = x_chunk_bytes(VAR);    // one chunk of streamed x
   using Geom = GeomOf<VAR>;
   constexpr int SS = 4 * SC;  // 16-wide k steps per stage
+  constexpr bool kRatio = MT * NT > 8;  // accumulators in units of the group scale (no part sums)
   // The kernel has no static shared memory, so the dynamic window starts on a
   // 1 KB boundary, which the 128-byte-swizzled x boxes rely on (checked
   // below).  Offsets from this base stay compile-time friendly; a rounded-up
@@ -292,8 +307,10 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
         } else {
           const int ls0 = (s - res_stages) * Geom::kLrSteps;
           const int nl = min(Geom::kLrSteps, p.nls - ls0);
-          const bool last = (s == res_stages + lr_stages - 1);
-          const bool first_sc4 = kSC4 && s == res_stages;  // SC4 row scales ride on the first rank-r stage
+          // Narrow instances read the correction's row scales from the last
+          // rank-r stage; SC4 row scales ride on the first.
+          const bool last = !kRatio && s == res_stages + lr_stages - 1;
+          const bool first_sc4 = kSC4 && s == res_stages;
           mbar_arrive_expect_tx(&full[st], (uint32_t)(ntile * (nl * kLrStepBytes + (last ? kTileRows * 2 : 0) +
                                                                 (first_sc4 ? kTileRows * 2 : 0))));
           for (int t = 0; t < ntile; ++t) {
@@ -324,7 +341,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
   }
 
   // ---------------- consumer warps ----------------
-  const int tsel = warp / (8 / MT);              // tile of the unit
+  const int tsel = warp / (8 / MT);          // tile of the unit
   const int mi0 = (warp % (8 / MT)) * MT;    // first of the warp's m-tiles in that tile
   const int gq = lane >> 2, cq = lane & 3;
   const int ng = p.d_pad / p.g;
@@ -395,7 +412,8 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
   // Factors that undo the staging scale for this lane's two token columns.
   float2 unscale[NT];
 #pragma unroll
-  for (int nt = 0; nt < NT; ++nt) unscale[nt] = make_float2(tscale[8 * nt + 2 * cq], tscale[8 * nt + 2 * cq + 1]);
+  for (int nt = 0; nt < NT; ++nt)
+    unscale[nt] = make_float2(tscale[8 * nt + 2 * cq], tscale[8 * nt + 2 * cq + 1]);
   // B-fragment bases: token 8*nt + gq (clamped to the M rows held; the extra
   // columns are never stored), column 2*cq (+ 16 per k step, + 8 for b1).
   const uint16_t *xb[NT];
@@ -411,19 +429,54 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
   for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x) {
     const int ntile = min(TL, p.num_tiles - TL * unit);
     const bool active = tsel < ntile;
+    // Narrow instances (MT * NT <= 8) sum each quantisation group in part,
+    // starting from the group's bias term, and promote it into acc by the
+    // group scale at the group's end.  Wide instances have no registers for
+    // a second set: their accumulators hold the running sum in units of the
+    // current group's scale (each group starts by multiplying them by
+    // previous scale / this scale and adding the bias term, and the last
+    // group's scale multiplies the finished residual once).  There a zero
+    // group scale counts as 1: the pack stores zero codes for such groups.
     float acc[MT][NT][4];
-    float part[MT][NT][4];  // one group's sums; each group's first MMA starts from zero
+    float part[kRatio ? 1 : MT][kRatio ? 1 : NT][4];
+    float sp_lo[MT], sp_hi[MT];  // wide: the previous group's scale (rows gq, gq + 8)
 #pragma unroll
-    for (int a = 0; a < MT; ++a)
+    for (int a = 0; a < MT; ++a) {
+      sp_lo[a] = sp_hi[a] = 0.f;
 #pragma unroll
       for (int b = 0; b < NT; ++b)
 #pragma unroll
-        for (int c = 0; c < 4; ++c) acc[a][b][c] = part[a][b][c] = 0.f;
+        for (int c = 0; c < 4; ++c) acc[a][b][c] = 0.f;
+    }
+#pragma unroll
+    for (int a = 0; a < (kRatio ? 1 : MT); ++a)
+#pragma unroll
+      for (int b = 0; b < (kRatio ? 1 : NT); ++b)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) part[a][b][c] = 0.f;
+    // Row scales of the correction branch (A_w).  Wide instances read them
+    // here and run the correction's k steps on acc / s_a, multiplying back by
+    // s_a at the end (a zero scale counts as 1; the pack stores zero codes
+    // for such rows).  Narrow instances take them from the last rank-r stage.
+    float a_lo[MT], a_hi[MT];
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) a_lo[mt] = a_hi[mt] = 1.f;
+    if (kRatio && active && p.nls > p.nls_core) {
+      const int64_t rb = ((int64_t)TL * unit + tsel) * kTileRows + mi0 * 16 + gq;
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt) {
+        a_lo[mt] = fp16_bits_to_f32(p.s_a[rb + mt * 16]);
+        a_hi[mt] = fp16_bits_to_f32(p.s_a[rb + mt * 16 + 8]);
+        a_lo[mt] = a_lo[mt] == 0.f ? 1.f : a_lo[mt];
+        a_hi[mt] = a_hi[mt] == 0.f ? 1.f : a_hi[mt];
+      }
+    }
 
-    // Residual: INT4 codes, promoted per group.  With x resident, each warp
-    // copies its share of a stage (codes and group scales) to registers and
-    // releases the slot at once, so the producer can refill it while the warp
-    // computes; with x streamed, it releases the slot after its k steps.
+    // Residual: INT4 codes, one scale per row and group.  With x resident,
+    // each warp copies its share of a stage (codes and group scales) to
+    // registers and releases the slot at once, so the producer can refill it
+    // while the warp computes; with x streamed, it releases the slot after its
+    // k steps.
     constexpr int NGS = GS <= SS ? SS / GS : 1;  // groups whose scales a stage carries
     for (int s = 0; s < res_stages; ++s) {
       if (!mbar_wait_warp(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
@@ -461,10 +514,23 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
           for (int gi = 0; gi < NGS; ++gi)
 #pragma unroll
             for (int mt = 0; mt < MT; ++mt) {
-              s_lo[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16]);
-              s_hi[gi][mt] = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16 + 8]) * (kF16 ? 0.0625f : 1.f);  // fp16: x16
+              const float lo = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16]);
+              const float hi = fp16_bits_to_f32(sc[gi * kTileRows + mt * 16 + 8]);
+              s_lo[gi][mt] = kRatio && lo == 0.f ? 1.f : lo;
+              s_hi[gi][mt] = (kRatio && hi == 0.f ? 1.f : hi) * (kF16 ? 0.0625f : 1.f);  // fp16: x16
             }
         }
+        // Wide: from here s_lo/s_hi hold the ratios to the previous group's scale.
+#pragma unroll
+        for (int gi = 0; gi < (kRatio ? NGS : 0); ++gi)
+#pragma unroll
+          for (int mt = 0; mt < MT; ++mt) {
+            const float lo = s_lo[gi][mt], hi = s_hi[gi][mt];
+            s_lo[gi][mt] = __fdividef(sp_lo[mt], lo);
+            s_hi[gi][mt] = __fdividef(sp_hi[mt], hi);
+            sp_lo[mt] = lo;
+            sp_hi[mt] = hi;
+          }
       }
       const int st_done = st;
       if (!kStreamX || !active) {
@@ -518,20 +584,38 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
             }
           }
           // First k step of a group (compile-time when groups fit in a stage).
-          // Its MMAs start from the group's bias term instead of zero:
-          // nb = -(operand bias) * sum of x over the group, per token, for
-          // rows gq (bias 1032, or 136 for bf16) and gq + 8 (1152 or 136), so
-          // that the finished part is the exact-code dot product.
+          // Its MMAs start from the group's bias term nb = -(operand bias) *
+          // sum of x over the group, per token, for rows gq (bias 1032, or 136
+          // for bf16) and gq + 8 (1152 or 136), so that the group adds its
+          // exact-code dot product: narrow, part = nb (the MMA's C operand);
+          // wide, acc = acc * (previous scale / this scale) + nb.
           const bool first = GS <= SS ? (ks % GS == 0) : (ks == 0 && (s % (GS / SS)) == 0);
-          float2 nb_lo[NT], nb_hi[NT];
-          if (first) {
+          float2 nb_lo[kRatio ? 1 : NT], nb_hi[kRatio ? 1 : NT];
+          if (first && !kRatio) {
+            const int ggl = GS <= SS ? s * (SS / GS) + ks / GS : s / (GS / SS);
+#pragma unroll
+            for (int nt = 0; nt < (kRatio ? 1 : NT); ++nt) {
+              const int o = ggl * XT + 8 * nt + 2 * cq;
+              nb_lo[nt] = *reinterpret_cast<const float2 *>(xsum_s + o);
+              nb_hi[nt] = kStreamX ? nb_lo[nt] : *reinterpret_cast<const float2 *>(xsum_s + ng * XT + o);
+            }
+          }
+          if (first && kRatio) {
             const int ggl = GS <= SS ? s * (SS / GS) + ks / GS : s / (GS / SS);  // group index along d
+            const int gi = GS <= SS ? ks / GS : 0;                                // group within the stage
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
               const int o = ggl * XT + 8 * nt + 2 * cq;
-              nb_lo[nt] = *reinterpret_cast<const float2 *>(xsum_s + o);
+              const float2 nb_lo = *reinterpret_cast<const float2 *>(xsum_s + o);
               // bf16 operands carry one bias (136) on both row halves
-              nb_hi[nt] = kStreamX ? nb_lo[nt] : *reinterpret_cast<const float2 *>(xsum_s + ng * XT + o);
+              const float2 nb_hi = kStreamX ? nb_lo : *reinterpret_cast<const float2 *>(xsum_s + ng * XT + o);
+#pragma unroll
+              for (int mt = 0; mt < MT; ++mt) {
+                acc[mt][nt][0] = fmaf(acc[mt][nt][0], s_lo[gi][mt], nb_lo.x);
+                acc[mt][nt][1] = fmaf(acc[mt][nt][1], s_lo[gi][mt], nb_lo.y);
+                acc[mt][nt][2] = fmaf(acc[mt][nt][2], s_hi[gi][mt], nb_hi.x);
+                acc[mt][nt][3] = fmaf(acc[mt][nt][3], s_hi[gi][mt], nb_hi.y);
+              }
             }
           }
 #pragma unroll
@@ -545,26 +629,36 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
               unpack_int4x8_biased(word, a);
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
-              if (kF16) {
-                if (first)
-                  mma_f16_16816_c(part[mt][nt], a, b[nt][0], b[nt][1], nb_lo[nt], nb_hi[nt]);
+              if constexpr (kRatio) {
+                if (kF16)
+                  mma_f16_16816(acc[mt][nt], a, b[nt][0], b[nt][1]);
                 else
-                  mma_f16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
+                  mma_bf16_16816(acc[mt][nt], a, b[nt][0], b[nt][1]);
               } else {
-                if (first)
-                  mma_bf16_16816_c(part[mt][nt], a, b[nt][0], b[nt][1], nb_lo[nt], nb_hi[nt]);
-                else
-                  mma_bf16_16816(part[mt][nt], a, b[nt][0], b[nt][1]);
+                float (&pt)[4] = part[kRatio ? 0 : mt][kRatio ? 0 : nt];
+                if (kF16) {
+                  if (first)
+                    mma_f16_16816_c(pt, a, b[nt][0], b[nt][1], nb_lo[kRatio ? 0 : nt], nb_hi[kRatio ? 0 : nt]);
+                  else
+                    mma_f16_16816(pt, a, b[nt][0], b[nt][1]);
+                } else {
+                  if (first)
+                    mma_bf16_16816_c(pt, a, b[nt][0], b[nt][1], nb_lo[kRatio ? 0 : nt], nb_hi[kRatio ? 0 : nt]);
+                  else
+                    mma_bf16_16816(pt, a, b[nt][0], b[nt][1]);
+                }
               }
             }
           }
-          // Group boundary: compile-time inside a stage when GS <= SS; every
-          // GS/SS stages otherwise.
-          const bool boundary = GS <= SS ? ((ks + 1) % GS == 0) : (ks == SS - 1 && ((s + 1) % (GS / SS)) == 0);
-          if (boundary) {
-            const int gi = GS <= SS ? ks / GS : 0;  // group within the stage
+          // Narrow: group boundary (compile-time inside a stage when GS <= SS;
+          // every GS/SS stages otherwise): promote part by the group scale.
+          if constexpr (!kRatio) {
+            const bool boundary = GS <= SS ? ((ks + 1) % GS == 0) : (ks == SS - 1 && ((s + 1) % (GS / SS)) == 0);
+            if (boundary) {
+              const int gi = GS <= SS ? ks / GS : 0;  // group within the stage
 #pragma unroll
-            for (int mt = 0; mt < MT; ++mt) promote<NT>(acc[mt], part[mt], s_lo[gi][mt], s_hi[gi][mt]);
+              for (int mt = 0; mt < MT; ++mt) promote<NT>(acc[mt], part[mt], s_lo[gi][mt], s_hi[gi][mt]);
+            }
           }
         }
       }
@@ -574,15 +668,18 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
       }
     }
 
-    // Back to the hidden states' own scale (exact: powers of two).
+    // The last group's scale, and back to the hidden states' own scale
+    // (exact: powers of two).
 #pragma unroll
-    for (int a = 0; a < (kF16 ? MT : 0); ++a)
+    for (int a = 0; a < MT; ++a)
 #pragma unroll
       for (int b = 0; b < NT; ++b) {
-        acc[a][b][0] *= unscale[b].x;
-        acc[a][b][1] *= unscale[b].y;
-        acc[a][b][2] *= unscale[b].x;
-        acc[a][b][3] *= unscale[b].y;
+        const float ux = kF16 ? unscale[b].x : 1.f, uy = kF16 ? unscale[b].y : 1.f;
+        const float fl = kRatio ? sp_lo[a] : 1.f, fh = kRatio ? sp_hi[a] : 1.f;
+        acc[a][b][0] *= fl * ux;
+        acc[a][b][1] *= fl * uy;
+        acc[a][b][2] *= fh * ux;
+        acc[a][b][3] *= fh * uy;
       }
     // SC4 without rank-r branches: no stage carries the row scales; read them here.
     if (kSC4 && lr_stages == 0 && active) {
@@ -601,11 +698,12 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
     }
 
     // Rank-r branches as extra k steps (core: factor 1; correction: row scale
-    // of A_w), with the same copy-then-release of each stage.
+    // of A_w), with the same copy-then-release of each stage.  Narrow: part
+    // sums again, promoted at the end of each branch.
 #pragma unroll
-    for (int a = 0; a < MT; ++a)
+    for (int a = 0; a < (kRatio ? 1 : MT); ++a)
 #pragma unroll
-      for (int b = 0; b < NT; ++b)
+      for (int b = 0; b < (kRatio ? 1 : NT); ++b)
 #pragma unroll
         for (int c = 0; c < 4; ++c) part[a][b][c] = 0.f;
     for (int s = 0; s < lr_stages; ++s) {
@@ -616,9 +714,7 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
       if (!mbar_wait_warp(&full[st], ph, p.wait_budget, abort_flag, p.err)) return;
       const int ls0 = s * Geom::kLrSteps;
       const int nl = min(Geom::kLrSteps, p.nls - ls0);
-      const bool last_stage = s == lr_stages - 1;
       uint2 lw[Geom::kLrSteps][MT];
-      float a_lo[MT], a_hi[MT];
       if (active) {
         const uint8_t *buf = smem + (size_t)st * Geom::kBytes;
 #pragma unroll
@@ -629,11 +725,13 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
               lw[l][mt] = *reinterpret_cast<const uint2 *>(
                   buf + ((size_t)(tsel * Geom::kLrSteps + l) * 8 + mi0 + mt) * 256 + lane * 8);
         const uint16_t *sa = reinterpret_cast<const uint16_t *>(buf + Geom::kCodeBytes + tsel * Geom::kScaleBytesPerTile);
+        if (!kRatio && s == lr_stages - 1) {
 #pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-          const int r = (mi0 + mt) * 16 + gq;
-          a_lo[mt] = last_stage ? fp16_bits_to_f32(sa[r]) : 0.f;
-          a_hi[mt] = last_stage ? fp16_bits_to_f32(sa[r + 8]) : 0.f;
+          for (int mt = 0; mt < MT; ++mt) {
+            const int r = (mi0 + mt) * 16 + gq;
+            a_lo[mt] = fp16_bits_to_f32(sa[r]);
+            a_hi[mt] = fp16_bits_to_f32(sa[r + 8]);
+          }
         }
         if (kSC4 && s == 0) {
           // The residual's row scales (SC4), before any rank-r term is added.
@@ -659,6 +757,19 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
       for (int l = 0; l < Geom::kLrSteps; ++l) {
         if (l >= nl) break;
         const int ls = ls0 + l;
+        if (kRatio && ls == p.nls_core) {  // first correction step: continue in units of s_a
+#pragma unroll
+          for (int mt = 0; mt < MT; ++mt) {
+            const float il = __fdividef(1.f, a_lo[mt]), ih = __fdividef(1.f, a_hi[mt]);
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+              acc[mt][nt][0] *= il;
+              acc[mt][nt][1] *= il;
+              acc[mt][nt][2] *= ih;
+              acc[mt][nt][3] *= ih;
+            }
+          }
+        }
         uint32_t bh[NT][2], bl[NT][2];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
@@ -677,22 +788,36 @@ __global__ void __launch_bounds__(kDecThreads, 1) decode_kernel(const __grid_con
           unpack_int8x8(lw[l][mt].x, lw[l][mt].y, a);
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
-            mma_bf16_16816(part[mt][nt], a, bh[nt][0], bh[nt][1]);
-            mma_bf16_16816(part[mt][nt], a, bl[nt][0], bl[nt][1]);
+            float (&pt)[4] = kRatio ? acc[mt][nt] : part[kRatio ? 0 : mt][kRatio ? 0 : nt];
+            mma_bf16_16816(pt, a, bh[nt][0], bh[nt][1]);
+            mma_bf16_16816(pt, a, bl[nt][0], bl[nt][1]);
           }
         }
-        if (ls + 1 == p.nls_core || ls + 1 == p.nls) {
-          const bool corr = ls + 1 == p.nls && p.nls > p.nls_core;  // the correction ends with the last stage
+        if constexpr (!kRatio) {
+          if (ls + 1 == p.nls_core || ls + 1 == p.nls) {
+            const bool corr = ls + 1 == p.nls && p.nls > p.nls_core;  // the correction ends with the last stage
 #pragma unroll
-          for (int mt = 0; mt < MT; ++mt) {
-            promote<NT>(acc[mt], part[mt], corr ? a_lo[mt] : 1.f, corr ? a_hi[mt] : 1.f);
+            for (int mt = 0; mt < MT; ++mt) {
+              promote<NT>(acc[mt], part[mt], corr ? a_lo[mt] : 1.f, corr ? a_hi[mt] : 1.f);
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt)
+              for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-              for (int c = 0; c < 4; ++c) part[mt][nt][c] = 0.f;
+                for (int c = 0; c < 4; ++c) part[mt][nt][c] = 0.f;
+            }
           }
         }
       }
+    }
+    if (kRatio && active && p.nls > p.nls_core) {  // the correction's row scale
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          acc[mt][nt][0] *= a_lo[mt];
+          acc[mt][nt][1] *= a_lo[mt];
+          acc[mt][nt][2] *= a_hi[mt];
+          acc[mt][nt][3] *= a_hi[mt];
+        }
     }
 
     // Epilogue.  acc[mt][nt][i]: row 16*(mi0+mt) + gq + 8*(i/2), token 8*nt + 2*cq + i%2.
@@ -793,7 +918,7 @@ static cudaError_t launch_t(const DecodeParams &dp, int grid, cudaStream_t s, co
   if (e != cudaSuccess || grid == 0) return e;  // grid 0: opt-in only (prepare_decode)
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(kDecThreads);
+  cfg.blockDim = dim3(variant_threads(VAR));
   cfg.dynamicSmemBytes = pl.total;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];

@@ -7,9 +7,12 @@
 namespace archead {
 
 // One block per (vocabulary tile, 64-wide chunk of d): stage the canonical
-// 128 x 32 bytes in shared memory, then emit the 1024 fragment words.
-__global__ void build_res_codes_kernel(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst, int64_t V, int d,
-                                       int d_pad) {
+// 128 x 32 bytes in shared memory, then emit the 1024 fragment words.  With
+// fp16 group scales given (INT8 format), the codes of a group whose scale is
+// zero are stored as zero: the weights are zero either way, and the decode
+// kernel relies on it (it runs such a group at scale 1).
+__global__ void build_res_codes_kernel(const uint8_t *__restrict__ src, const uint16_t *__restrict__ scales,
+                                       uint8_t *__restrict__ dst, int64_t V, int d, int d_pad, int G, int g) {
   __shared__ uint8_t tile[kTileRows][kChunkK / 2];
   const int KC = d_pad / kChunkK;
   const int vt = blockIdx.x / KC;
@@ -18,7 +21,9 @@ __global__ void build_res_codes_kernel(const uint8_t *__restrict__ src, uint8_t 
     int r = i / (kChunkK / 2), b = i % (kChunkK / 2);
     int64_t row = (int64_t)vt * kTileRows + r;
     // Padding rows and padding columns (k >= d; d is a multiple of 64) hold code 0.
-    tile[r][b] = (row < V && kc * kChunkK < d) ? src[row * (d / 2) + (int64_t)kc * (kChunkK / 2) + b] : (uint8_t)0;
+    const int k = kc * kChunkK + 2 * b;
+    const bool zero_scale = scales != nullptr && row < V && k < d && (scales[row * G + k / g] & 0x7FFFu) == 0;
+    tile[r][b] = (row < V && k < d && !zero_scale) ? src[row * (d / 2) + (int64_t)kc * (kChunkK / 2) + b] : (uint8_t)0;
   }
   __syncthreads();
   uint32_t *out = reinterpret_cast<uint32_t *>(dst) + ((int64_t)vt * KC + kc) * 1024;
@@ -77,8 +82,11 @@ __device__ __forceinline__ int int5_code(const uint8_t *row, int j) {
 
 // One block per (tile, 16-wide step of the extended rank axis).  core_u is
 // int8 [V][r_c], or with u5 != 0 the SC4 5-bit codes [V][ceil(5 r_c / 8)].
+// A correction row whose scale is zero is stored as zero codes (its weights
+// are zero either way; the decode kernel runs it at scale 1).
 __global__ void build_lr_codes_kernel(const void *__restrict__ core_u, const int8_t *__restrict__ corr_a,
-                                      uint8_t *__restrict__ dst, int64_t V, int rc, int rr, int rcp, int nls, int u5) {
+                                      const uint16_t *__restrict__ corr_a_scale, uint8_t *__restrict__ dst, int64_t V,
+                                      int rc, int rr, int rcp, int nls, int u5) {
   const int vt = blockIdx.x / nls;
   const int ls = blockIdx.x % nls;
   uint8_t *out = dst + ((int64_t)vt * nls + ls) * kLrStepBytes;
@@ -94,7 +102,7 @@ __global__ void build_lr_codes_kernel(const void *__restrict__ core_u, const int
         if (kk < rc)
           code = u5 ? int5_code(static_cast<const uint8_t *>(core_u) + row * ((5 * rc + 7) / 8), kk)
                     : static_cast<const int8_t *>(core_u)[row * rc + kk];
-      } else if (kk - rcp < rr) {
+      } else if (kk - rcp < rr && (corr_a_scale[row] & 0x7FFFu) != 0) {
         code = corr_a[row * rr + (kk - rcp)];
       }
     }
@@ -131,7 +139,8 @@ cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, cons
                                  const uint16_t *row_scale, const void *core_u, const int8_t *corr_a,
                                  const uint16_t *corr_a_scale, cudaStream_t s) {
   const int KC = p->d_pad / kChunkK;
-  build_res_codes_kernel<<<p->num_tiles * KC, 256, 0, s>>>(res_codes, p->codes, p->V, p->d, p->d_pad);
+  build_res_codes_kernel<<<p->num_tiles * KC, 256, 0, s>>>(
+      res_codes, p->sc4 ? nullptr : static_cast<const uint16_t *>(res_scales), p->codes, p->V, p->d, p->d_pad, p->G, p->g);
   if (p->sc4) {
     build_scale_codes_kernel<<<1024, 256, 0, s>>>(static_cast<const uint8_t *>(res_scales), p->scodes, p->V, p->V_pad,
                                                   p->G, p->G_pad2);
@@ -141,8 +150,8 @@ cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, cons
                                                  p->G, p->G_pad);
   }
   if (p->nls > 0)
-    build_lr_codes_kernel<<<p->num_tiles * p->nls, 256, 0, s>>>(core_u, corr_a, p->lr_codes, p->V, p->rc, p->rr,
-                                                                 p->rcp, p->nls, p->sc4);
+    build_lr_codes_kernel<<<p->num_tiles * p->nls, 256, 0, s>>>(core_u, corr_a, corr_a_scale, p->lr_codes, p->V, p->rc,
+                                                                 p->rr, p->rcp, p->nls, p->sc4);
   build_row_scales_kernel<<<256, 256, 0, s>>>(p->rr > 0 ? corr_a_scale : nullptr, p->s_a, p->V, p->V_pad);
   if (p->lr > 0)
     build_lr_t_kernel<<<256, 256, 0, s>>>(p->q_v, p->q_b, p->lr_t, p->d, p->d_pad, p->rc, p->rr, p->rcp, p->lr);

@@ -9,7 +9,8 @@
   every path, and the lowest vocabulary row wins; an all-zero head gives
   CE = log V and near-zero logits;
 - cross entropy far from logit rms 2: one dominant row (CE from ~0 to far
-  above log V) and hidden states scaled by 2^3, 2^6 and 2^10.
+  above log V) and hidden states scaled by 2^3, 2^6 and 2^10;
+- zero group, row and correction scales (+0 and -0).
 """
 
 import math
@@ -150,6 +151,56 @@ def test_ragged_token_tiles_ce_and_greedy(name, M):
         assert np.all(err <= gu.CE_ABS), f"{name} M={M} path={path}: max|dCE|={err.max():.3e}"
         idx, val = gu.forward_argmax(pack, x, path)
         gu.check_greedy(idx, val, ref_y, where=f"{name} M={M} path={path}")
+
+
+# ---------------------------------------------------------------------------
+# Zero scales
+# ---------------------------------------------------------------------------
+def _zero_scale_head(shape, seed):
+    """About one in eight residual group scales (INT8 format) or row scales
+    (SC4) set to +0 or -0, one whole row of them, and as many correction row
+    scales.  Their weights are zero whatever the codes; the pack stores zero
+    codes there, and the 64-token decode instance runs such groups at scale 1."""
+    head = make_head(shape, seed=seed)
+    rng = np.random.default_rng(seed)
+    key = "res_row_scale" if shape.fmt == "sc4" else "res_scales"
+    s = head[key]
+    mask = rng.random(s.shape) < 0.125
+    s[mask] = np.where(rng.random(int(mask.sum())) < 0.5, 0x0000, 0x8000).astype(np.uint16)
+    s[3] = 0
+    if shape.corr_rank:
+        a = head["corr_a_scale"]
+        a[rng.random(a.shape) < 0.125] = 0
+        a[5] = 0x8000
+    return head
+
+
+@pytest.mark.parametrize("name", ["tiny", "g32", "g128", "max_rank", "sc4", "sc4_g32"])
+def test_zero_scales(name):
+    """Zero group, row and correction scales against the oracle: logits on
+    every path at the token counts of every decode instance, and the
+    dequantised components (equal as numbers: a zero weight may come back
+    as +0 where the oracle's product is -0)."""
+    import torch
+
+    shape = SHAPES[name]
+    head = _zero_scale_head(shape, seed=_seed(name) + 1)
+    pack = archead.archead_pack_create(head, shape)
+    try:
+        comps = [("residual", shape.V, shape.d)] + ([("corr_a", shape.V, shape.corr_rank)] if shape.corr_rank else [])
+        for comp, rows, cols in comps:
+            out = torch.full((rows, cols), float("nan"), dtype=torch.float32, device="cuda")
+            archead.archead_debug_dequant(pack, comp, 0, rows, out)
+            torch.cuda.synchronize()
+            assert np.array_equal(out.cpu().numpy().astype(np.float64), oracle.component(head, shape, comp)), comp
+        x = make_hidden(shape.d, 64, seed=31)
+        ref = oracle.logits(head, shape, x)
+        for M in (1, 9, 16, 27, 40, 64):
+            for path in PATHS:
+                got = gu.forward(pack, x[:M], archead.OUT_FP32, path)
+                gu.check_logits(got, ref[:M], where=f"{name} zero scales M={M} path={path}")
+    finally:
+        pack.close()
 
 
 # ---------------------------------------------------------------------------
