@@ -50,7 +50,9 @@ constexpr int kSmemLimit = 227 * 1024;
 //    16 tokens, loaded by a 2-D TMA copy, and the operands stay bf16 (no fp16
 //    staging).  Its warps read codes and x from the stage as they compute and
 //    release it afterwards (the registers to copy a stage out first are not
-//    there with two n-tiles).
+//    there with two n-tiles).  Sixteen consumer warps of two m-tiles each
+//    (92.1 us at M = 16 against 94.2 with eight warps of four; for M <= 8 the
+//    resident instance keeps eight warps: 67.7 against 73.8 us with sixteen).
 // Measured alternatives that were slower on the Qwen3-8B-shaped head (and not
 // kept): 16 tokens of x resident as fp16 with a 2-chunk ring (98.4 us at
 // M = 16 against 94.8) or a 1-chunk ring with the next stage prefetched into
@@ -73,9 +75,11 @@ enum DecodeVariant { kDecResident1 = 0, kDecStreamed2 = 1, kDecWide4 = 2, kDecWi
 __host__ __device__ constexpr int variant_nt(int v) {  // 8-token n-tiles
   return v == kDecResident1 ? 1 : v == kDecStreamed2 ? 2 : v == kDecWide4 ? 4 : 8;
 }
-__host__ __device__ constexpr int variant_cw(int v) { return v == kDecWide4 ? 16 : 8; }  // consumer warps
+__host__ __device__ constexpr int variant_cw(int v) {  // consumer warps
+  return v == kDecResident1 || v == kDecWide8 ? 8 : 16;
+}
 __host__ __device__ constexpr int variant_mt(int v) {  // 16-row m-tiles per consumer warp
-  return v == kDecWide4 ? 1 : v == kDecWide8 ? 2 : 4;
+  return v == kDecResident1 ? 4 : v == kDecWide4 ? 1 : 2;
 }
 // 128-row tiles per unit: the consumer warps cover them, MT m-tiles each.
 __host__ __device__ constexpr int variant_tiles(int v) { return variant_cw(v) * variant_mt(v) / 8; }
