@@ -501,6 +501,10 @@ def flat_keys(result):
             if mode in bp:
                 out[f"{name}_prefill_m{bp['M']}_{mode}_ms"] = bp[mode]["ms_per_call"]
                 out[f"{name}_prefill_m{bp['M']}_{mode}_frac_bf16_peak"] = bp[mode]["frac_bf16_peak"]
+    for row in (result.get("crossover") or {}).get("rows") or []:
+        if row["M"] in (32, 64, 256, 4096):
+            out[f"qwen_crossover_m{row['M']}_auto_us"] = row["auto_us"]
+            out[f"qwen_crossover_m{row['M']}_dense_bf16_us"] = row["dense_bf16_us"]
     c = result.get("construct") or {}
     if "seconds" in c:
         out["construct_qwen_sc4_seconds"] = c["seconds"]
@@ -585,9 +589,10 @@ def prefill_block(pack, shape, peaks, world, local_rank, M=4096):
 
 
 def crossover_sweep(pack, shape, world, local_rank):
-    """Batch sweep on one head: per M the decode kernel (tokens 16 at a time),
-    the prefill kernel, the automatic choice and a dense BF16 cuBLAS GEMM of
-    the same shape, each as microseconds per call (bf16 logits out)."""
+    """Batch sweep on one head: per M the decode kernel (one launch per 16,
+    32 or 64 tokens), the prefill kernel, the automatic choice and a dense
+    BF16 cuBLAS GEMM of the same shape, each as microseconds per call (bf16
+    logits out)."""
     import torch
 
     from paper_2608_02703_gb300 import archead
@@ -598,7 +603,7 @@ def crossover_sweep(pack, shape, world, local_rank):
     W = (torch.randn((shape.V, shape.d), generator=g, device="cuda", dtype=torch.float32) * 0.01).to(torch.bfloat16)
     dev = torch.device("cuda", local_rank)
     rows = []
-    for M in (1, 4, 16, 64, 256, 1024, 4096, 8192):
+    for M in (1, 4, 16, 32, 64, 128, 256, 1024, 4096, 8192):
         x = torch.from_numpy(make_hidden(shape.d, M, seed=5, n_outliers=shape.n_outliers).view(np.int16)).cuda()
         y = torch.empty((M, shape.V), dtype=torch.bfloat16, device="cuda")
         k = 200 if M <= 16 else (20 if M <= 1024 else 4)
