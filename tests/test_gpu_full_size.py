@@ -1,7 +1,8 @@
 """Full-size heads (the Qwen3-8B and Gemma-shaped configurations and the
 Qwen3-8B head in the paper's own packed format, the same seeded heads
 bench.py times) through the C ABI against the fp64 oracle:
-the whole vocabulary for decode token counts, sampled tokens for prefill
+the whole vocabulary for decode token counts (all tokens up to 16, sampled
+tokens of the 32- and 64-token launches), sampled tokens for prefill
 (a token's logits depend on that token's hidden state only, so the oracle
 checks sampled rows exactly)."""
 
@@ -83,6 +84,36 @@ def test_greedy_full_vocabulary(name):
     ref = oracle.logits(head, shape, x)
     idx, val = gu.forward_argmax(pack, x)
     gu.check_greedy(idx, val, ref, where=f"{name} greedy M={M}")
+
+
+@pytest.mark.parametrize("name", FULL)
+@pytest.mark.parametrize("M", [27, 64])
+def test_decode_wide_sampled_tokens(name, M):
+    """One launch of the 32- resp. 64-token decode instance (every n-tile of
+    the launch, the ragged one included) over the whole vocabulary: logits,
+    greedy output and fused CE on one token of each 8-token n-tile."""
+    import torch
+
+    pack, head = get(name)
+    shape = SHAPES[name]
+    x = make_hidden(shape.d, M, seed=4, n_outliers=shape.n_outliers)
+    t = make_targets(shape.V, M, seed=4)
+    idx = np.unique(np.minimum(np.arange(0, M + 7, 8) + (np.arange(0, M + 7, 8) // 8) % 8, M - 1))
+    ref = oracle.logits(head, shape, x[idx])
+    y = torch.full((M, shape.V), float("nan"), dtype=torch.float32, device="cuda")
+    archead.archead_forward(pack, gu.to_dev(x), M, y, archead.OUT_FP32)
+    assert archead.archead_sync_status(pack) == archead.OK
+    got = _rows(y, torch.from_numpy(idx).cuda())
+    gu.check_logits(got, ref, where=f"{name} decode M={M} sampled")
+    gu.check_argmax(got, ref, where=f"{name} decode M={M} sampled")
+    del y
+    gi, gv = gu.forward_argmax(pack, x)
+    gu.check_greedy(gi[idx], gv[idx], ref, where=f"{name} decode greedy M={M} sampled")
+    ce, st = gu.forward_ce(pack, x, t)
+    assert st == archead.OK
+    ref_ce = oracle.cross_entropy(head, shape, x[idx], t[idx])
+    d = np.abs(ce[idx] - ref_ce["ce"])
+    assert np.max(d) <= gu.CE_ABS, f"{name}: decode CE M={M} max|d|={np.max(d):.3e}"
 
 
 @pytest.mark.parametrize("name", FULL)
