@@ -25,7 +25,10 @@
  *  - Device pointers must be 16-byte aligned; x rows must be contiguous.
  *  - A pack may be used by one stream at a time (the workspace it owns for
  *    the pre-pass and the cross-entropy partials is not shared safely between
- *    concurrent calls).  Different packs are independent.
+ *    concurrent calls); successive calls may use different streams.  When a
+ *    call needs a larger workspace than the pack holds, it synchronises the
+ *    device before freeing the old one, so earlier calls on any stream are
+ *    done with it.  Different packs are independent.
  *  - Faults detected on the device (an out-of-range target, a pipeline wait
  *    that gave up) are latched in a per-pack device error word and reported
  *    by archead_sync_status().
@@ -35,6 +38,10 @@
 
 #include <stddef.h>
 #include <stdint.h>
+
+/* Version of this interface: 2 added archead_pack_create_ex and
+ * archead_abi_version.  archead_desc only grows by appending fields. */
+#define ARCHEAD_ABI_VERSION 2
 
 #if defined(__GNUC__)
 #define ARCHEAD_API __attribute__((visibility("default")))
@@ -147,6 +154,20 @@ typedef struct {
  * buffers may be freed as soon as it returns.  On failure *out is NULL.
  */
 ARCHEAD_API archead_status archead_pack_create(const archead_desc *desc, void *stream, archead_pack **out);
+
+/*
+ * archead_pack_create with the caller's sizeof(archead_desc).  The library
+ * reads only the fields that lie within desc_size, so a struct compiled
+ * against an older header (appended fields missing) stays valid; the fields
+ * of version 1 (up to corr_b_scale) are required (ARCHEAD_ERR_INVALID_ARG if
+ * desc_size is smaller), and a field the format needs that lies beyond
+ * desc_size (res_row_scale for ARCHEAD_FORMAT_SC4) is ARCHEAD_ERR_INVALID_ARG.
+ */
+ARCHEAD_API archead_status archead_pack_create_ex(const archead_desc *desc, size_t desc_size, void *stream,
+                                                  archead_pack **out);
+
+/* ARCHEAD_ABI_VERSION of the library actually loaded. */
+ARCHEAD_API int archead_abi_version(void);
 
 /* Free a pack and everything it owns.  NULL is a no-op. */
 ARCHEAD_API void archead_destroy(archead_pack *pack);

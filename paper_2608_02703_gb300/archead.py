@@ -45,7 +45,7 @@ EXPORTED = (
     "archead_forward_decode_noalloc", "archead_forward_argmax", "archead_forward_argmax_path",
     "archead_forward_lse_partial", "archead_lse_combine", "archead_argmax_combine",
     "archead_quantize_symmetric", "archead_quantize_residual_sc4", "archead_pack_codes", "archead_dequant_symmetric",
-    "archead_dequant_residual_sc4",
+    "archead_dequant_residual_sc4", "archead_pack_create_ex", "archead_abi_version",
 )
 
 
@@ -95,6 +95,8 @@ def load() -> ctypes.CDLL:
     vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
     sig = {
         "archead_pack_create": (i32, [ctypes.POINTER(archead_desc), vp, ctypes.POINTER(vp)]),
+        "archead_pack_create_ex": (i32, [ctypes.POINTER(archead_desc), ctypes.c_size_t, vp, ctypes.POINTER(vp)]),
+        "archead_abi_version": (i32, []),
         "archead_destroy": (None, [vp]),
         "archead_forward": (i32, [vp, vp, i64, vp, i32, vp]),
         "archead_forward_path": (i32, [vp, vp, i64, vp, i32, i32, vp]),
@@ -179,12 +181,13 @@ class Pack:
             self.handle = None
 
 
-def archead_pack_create(head: Dict, shape, stream=None) -> Pack:
+def archead_pack_create(head: Dict, shape, stream=None, desc_size=None) -> Pack:
     """Build a pack from canonical arrays (numpy host arrays or torch tensors).
 
     The INT8 format takes the arrays named as the struct fields; the paper's
     format (shape.fmt == "sc4") takes res_scale_codes, res_row_scale and
-    core_u5 in place of res_scales and core_u."""
+    core_u5 in place of res_scales and core_u.  With desc_size the call goes
+    through archead_pack_create_ex with that struct size."""
     sc4 = getattr(shape, "fmt", "int8") == "sc4"
     d = archead_desc(vocab=shape.V, hidden=shape.d, core_rank=shape.core_rank, corr_rank=shape.corr_rank,
                      group_size=shape.group_size, format=FORMAT_SC4 if sc4 else FORMAT_INT8)
@@ -200,8 +203,16 @@ def archead_pack_create(head: Dict, shape, stream=None) -> Pack:
         keep.append(a)
         setattr(d, name, _ptr(a) if a is not None and getattr(a, "size", 1) != 0 else None)
     h = ctypes.c_void_p()
-    _check(load().archead_pack_create(ctypes.byref(d), _stream_ptr(stream), ctypes.byref(h)), "archead_pack_create")
+    if desc_size is None:
+        _check(load().archead_pack_create(ctypes.byref(d), _stream_ptr(stream), ctypes.byref(h)), "archead_pack_create")
+    else:
+        _check(load().archead_pack_create_ex(ctypes.byref(d), desc_size, _stream_ptr(stream), ctypes.byref(h)),
+               "archead_pack_create_ex")
     return Pack(h.value, shape)
+
+
+def archead_abi_version() -> int:
+    return int(load().archead_abi_version())
 
 
 def archead_destroy(pack: Pack) -> None:

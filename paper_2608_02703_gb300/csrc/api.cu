@@ -3,6 +3,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cstddef>
 #include <cstring>
 #include <map>
 #include <mutex>
@@ -67,9 +68,12 @@ struct Carve {
   }
 };
 
+// Growing a buffer synchronises the device, not only the caller's stream:
+// a call made earlier on another stream may still be using the old one.
 cudaError_t ensure_workspace(archead_pack *p, size_t bytes, cudaStream_t s) {
+  (void)s;
   if (bytes <= p->ws_bytes) return cudaSuccess;
-  cudaError_t e = cudaStreamSynchronize(s);
+  cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return e;
   if (p->ws) {
     cudaFree(p->ws);
@@ -88,8 +92,9 @@ cudaError_t ensure_workspace(archead_pack *p, size_t bytes, cudaStream_t s) {
 // Block counters of the pre-pass: zeroed once when (re)allocated; every
 // pre-pass call leaves them zero again.
 cudaError_t ensure_counters(archead_pack *p, int n, cudaStream_t s) {
+  (void)s;
   if (n <= p->counters_len) return cudaSuccess;
-  cudaError_t e = cudaStreamSynchronize(s);
+  cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return e;
   if (p->counters) {
     cudaFree(p->counters);
@@ -361,6 +366,18 @@ void timer_end(archead_pack *p, const char *name, cudaStream_t s, cudaEvent_t ev
 
 extern "C" {
 
+int archead_abi_version(void) { return ARCHEAD_ABI_VERSION; }
+
+archead_status archead_pack_create_ex(const archead_desc *desc, size_t desc_size, void *stream, archead_pack **out) {
+  if (!out) return ARCHEAD_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!desc || desc_size < offsetof(archead_desc, res_row_scale)) return ARCHEAD_ERR_INVALID_ARG;
+  // Fields past the caller's struct read as zero (absent).
+  archead_desc d{};
+  std::memcpy(&d, desc, std::min(desc_size, sizeof(archead_desc)));
+  return archead_pack_create(&d, stream, out);
+}
+
 archead_status archead_pack_create(const archead_desc *desc, void *stream, archead_pack **out) {
   if (!out) return ARCHEAD_ERR_INVALID_ARG;
   *out = nullptr;
@@ -572,7 +589,7 @@ archead_status archead_forward_host(archead_pack *pack, const void *x_host, int6
   cudaGetLastError();  // a pointer the runtime does not know is not an error here
   const size_t need_y = y_direct ? 0 : yb;
   if (xb > pack->xh_bytes || need_y > pack->yh_bytes) {
-    AH_CUDA(cudaStreamSynchronize(s));
+    AH_CUDA(cudaDeviceSynchronize());  // earlier calls on any stream are done with the old buffers
     if (xb > pack->xh_bytes) {
       if (pack->xh_dev) cudaFree(pack->xh_dev), pack->owned_bytes -= (int64_t)pack->xh_bytes;
       pack->xh_dev = nullptr;

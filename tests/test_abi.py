@@ -66,6 +66,29 @@ def test_pack_create_rejects_bad_desc(lib, bad):
     assert out.value is None
 
 
+def test_abi_version(lib):
+    with open(os.path.join(INCLUDE, "archead.h")) as f:
+        declared = int(re.search(r"#define ARCHEAD_ABI_VERSION (\d+)", f.read()).group(1))
+    assert lib.archead_abi_version() == declared == archead.archead_abi_version() == 2
+
+
+def test_pack_create_ex_reads_only_the_callers_struct(lib):
+    """A struct of version 1 (up to corr_b_scale) is accepted for the INT8
+    format; fields past desc_size read as absent even if the memory behind
+    them is set, so the paper's format (which needs res_row_scale) is
+    refused; a struct shorter than version 1 is refused."""
+    v1 = archead.archead_desc.res_row_scale.offset
+    out = ctypes.c_void_p(1234)
+    assert lib.archead_pack_create_ex(ctypes.byref(_desc()), v1 - 8, None, ctypes.byref(out)) == archead.ERR_INVALID_ARG
+    assert out.value is None
+    assert lib.archead_pack_create_ex(None, v1, None, ctypes.byref(out)) == archead.ERR_INVALID_ARG
+    sc4 = _desc(format=1)  # res_row_scale set, but past the size given
+    assert lib.archead_pack_create_ex(ctypes.byref(sc4), v1, None, ctypes.byref(out)) == archead.ERR_INVALID_ARG
+    # A version-1 INT8 struct reaches the shape checks (an invalid shape is reported as such).
+    assert lib.archead_pack_create_ex(ctypes.byref(_desc(hidden=100)), v1, None,
+                                      ctypes.byref(out)) == archead.ERR_INVALID_ARG
+
+
 def test_pack_create_null_args(lib):
     out = ctypes.c_void_p()
     assert lib.archead_pack_create(None, None, ctypes.byref(out)) == archead.ERR_INVALID_ARG

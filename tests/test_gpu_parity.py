@@ -57,6 +57,25 @@ def get(name):
     return _packs[name]
 
 
+def test_pack_create_ex_version1_struct():
+    """An INT8 head described by a version-1 struct (no res_row_scale)
+    through archead_pack_create_ex gives the same logits as the full struct."""
+    import ctypes
+
+    pack, head = get("tiny")
+    shape = SHAPES["tiny"]
+    v1 = archead.archead_desc.res_row_scale.offset
+    old = archead.archead_pack_create(head, shape, desc_size=v1)
+    try:
+        x = make_hidden(shape.d, 9, seed=21)
+        a = gu.forward(pack, x, archead.OUT_FP32, archead.PATH_AUTO)
+        b = gu.forward(old, x, archead.OUT_FP32, archead.PATH_AUTO)
+        assert np.array_equal(a, b)
+        assert ctypes.sizeof(archead.archead_desc) > v1
+    finally:
+        old.close()
+
+
 @pytest.mark.parametrize("name", sorted(SHAPES))
 def test_dequant_bit_exact(name):
     import torch
