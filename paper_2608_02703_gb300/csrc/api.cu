@@ -45,7 +45,8 @@ cudaError_t dev_alloc(archead_pack *p, T **ptr, size_t bytes) {
 
 void free_pack(archead_pack *p) {
   if (!p) return;
-  void *bufs[] = {p->codes, p->scales, p->scodes, p->s_row,  p->lr_codes, p->s_a,    p->q_v,
+  if (p->lr_codes_dec == p->lr_codes) p->lr_codes_dec = nullptr;  // the same buffer
+  void *bufs[] = {p->codes, p->scales, p->scodes, p->s_row,  p->lr_codes, p->lr_codes_dec, p->s_a,    p->q_v,
                   p->q_b,   p->lr_t,   p->s_u,    p->s_v,    p->s_b,      p->err,    p->ws,
                   p->xh_dev, p->yh_dev, p->counters};
   for (void *b : bufs)
@@ -123,12 +124,12 @@ struct ForwardPlan {
 ForwardPlan plan_decode(archead_pack *p, int64_t M, bool ce) {
   ForwardPlan f;
   Carve c;
-  f.variant = decode_variant(p->d_pad, p->nls, p->g, (int)std::min<int64_t>(M, kDecodeWideTokens));
+  f.variant = decode_variant(p->d_pad, p->nls_dec, p->g, (int)std::min<int64_t>(M, kDecodeWideTokens));
   f.chunk_tokens = decode_variant_tokens(f.variant);
   f.nchunks = (int)((M + f.chunk_tokens - 1) / f.chunk_tokens);
   f.partial_off = c.take(prepass_partial_bytes((int)M, p->lr, p->d));
   // rank-r fragments, in 16-token chunks
-  f.ts_off = c.take((size_t)((M + kDecodeMaxTokens - 1) / kDecodeMaxTokens) * std::max(p->nls, 1) * 1024);
+  f.ts_off = c.take((size_t)((M + kDecodeMaxTokens - 1) / kDecodeMaxTokens) * std::max(p->nls_dec, 1) * 1024);
   if (ce) {
     f.ce_part_off = c.take((size_t)decode_num_units(p, f.variant) * decode_parts_per_unit(f.variant) * M * sizeof(float2));
     f.tlogit_off = c.take((size_t)M * sizeof(float));
@@ -155,7 +156,7 @@ archead_status check_forward_args(archead_pack *p, const void *x, int64_t M, con
 archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, int out_fp32,
                           const int32_t *targets, float *ce, int32_t *amax_idx, float *amax_val, int row0,
                           float *parts3, cudaStream_t s) {
-  if (!decode_supported(p->d_pad, p->nls, p->g)) return ARCHEAD_ERR_UNSUPPORTED;
+  if (!decode_supported(p->d_pad, p->nls_dec, p->g)) return ARCHEAD_ERR_UNSUPPORTED;
   const bool ce_mode = out == nullptr;
   const bool greedy = amax_idx != nullptr;
   ForwardPlan f = plan_decode(p, M, ce_mode);
@@ -182,7 +183,7 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   for (int c = 0; c < f.nchunks; ++c) {
     dp.m0 = c * f.chunk_tokens;
     dp.M = (int)std::min<int64_t>(f.chunk_tokens, M - dp.m0);
-    dp.ts = pp.ts + (size_t)(dp.m0 / kDecodeMaxTokens) * p->nls * 256;
+    dp.ts = pp.ts + (size_t)(dp.m0 / kDecodeMaxTokens) * p->nls_dec * 256;
     cudaEvent_t ev = nullptr;
     timer_begin(p, "decode", s, &ev);
     // The first chunk overlaps the pre-pass grid (programmatic dependent launch).
@@ -261,8 +262,8 @@ archead_status run_forward(archead_pack *p, const void *x, int64_t M, void *out,
   // sums of x for 16 tokens, e.g. d = 2^20 at g = 32) take the prefill
   // kernel under AUTO.
   bool decode = path == ARCHEAD_PATH_DECODE;
-  if (path == ARCHEAD_PATH_AUTO && M <= kDecodeWideTokens && decode_supported(p->d_pad, p->nls, p->g)) {
-    const int tok = decode_variant_tokens(decode_variant(p->d_pad, p->nls, p->g, (int)M));
+  if (path == ARCHEAD_PATH_AUTO && M <= kDecodeWideTokens && decode_supported(p->d_pad, p->nls_dec, p->g)) {
+    const int tok = decode_variant_tokens(decode_variant(p->d_pad, p->nls_dec, p->g, (int)M));
     decode = (M + tok - 1) / tok <= 3;
   }
   if (decode) return run_decode(p, x, M, out, out_fp32, targets, ce, amax_idx, amax_val, row0, parts3, s);
@@ -291,6 +292,9 @@ PrepassParams prepass_params(const archead_pack *p, const void *x, int64_t M) {
   pp.rcp = p->rcp;
   pp.rrp = p->rrp;
   pp.lr = p->lr;
+  pp.ts_nls = p->nls_dec;
+  pp.ts_core = p->core_cols;
+  pp.ts_compact = p->nls_dec < p->nls;
   return pp;
 }
 
@@ -302,7 +306,7 @@ DecodeParams decode_params(const archead_pack *p, const void *x, int64_t M_total
   dp.s_row = p->s_row;
   dp.sc4 = p->sc4;
   dp.G_pad2 = p->G_pad2;
-  dp.lr_codes = p->lr_codes;
+  dp.lr_codes = p->lr_codes_dec;
   dp.s_a = p->s_a;
   dp.x = static_cast<const uint16_t *>(x);
   dp.V = p->V;
@@ -311,8 +315,9 @@ DecodeParams decode_params(const archead_pack *p, const void *x, int64_t M_total
   dp.d_pad = p->d_pad;
   dp.G_pad = p->G_pad;
   dp.g = p->g;
-  dp.nls = p->nls;
-  dp.nls_core = p->nls_core;
+  dp.nls = p->nls_dec;
+  dp.core_cols = p->core_cols;
+  dp.has_corr = p->rr > 0;
   dp.M_total = (int)M_total;
   dp.err = p->err;
   dp.wait_budget = p->wait_budget;
@@ -433,6 +438,16 @@ archead_status archead_pack_create(const archead_desc *desc, void *stream, arche
   p->lr = p->rcp + p->rrp;
   p->nls = p->lr / 16;
   p->nls_core = p->rcp / 16;
+  // The decode kernel's rank-r steps in the paper's format: both branches
+  // back to back, padded once (its r_c = 10, r_r = 6 fit one 16-wide step
+  // instead of two).  The INT8 format keeps each branch padded to 16.
+  if (sc4 && (rc + rr + 15) / 16 < p->nls) {
+    p->nls_dec = (rc + rr + 15) / 16;
+    p->core_cols = rc;
+  } else {
+    p->nls_dec = p->nls;
+    p->core_cols = p->rcp;
+  }
 
   const size_t G = p->G;
   if ((e = dev_alloc(p, &p->codes, (size_t)p->V_pad * p->d_pad / 2)) != cudaSuccess) return fail(e);
@@ -443,6 +458,12 @@ archead_status archead_pack_create(const archead_desc *desc, void *stream, arche
     if ((e = dev_alloc(p, &p->scales, (size_t)p->V_pad * p->G_pad * 2)) != cudaSuccess) return fail(e);
   }
   if ((e = dev_alloc(p, &p->lr_codes, (size_t)p->num_tiles * p->nls * kLrStepBytes)) != cudaSuccess) return fail(e);
+  if (p->nls_dec < p->nls) {
+    if ((e = dev_alloc(p, &p->lr_codes_dec, (size_t)p->num_tiles * p->nls_dec * kLrStepBytes)) != cudaSuccess)
+      return fail(e);
+  } else {
+    p->lr_codes_dec = p->lr_codes;
+  }
   if ((e = dev_alloc(p, &p->s_a, (size_t)p->V_pad * 2)) != cudaSuccess) return fail(e);
   if ((e = dev_alloc(p, &p->q_v, (size_t)d * rc)) != cudaSuccess) return fail(e);
   if ((e = dev_alloc(p, &p->q_b, (size_t)d * rr)) != cudaSuccess) return fail(e);

@@ -48,10 +48,10 @@ cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool
 // Opt in every instance the pack can launch: the largest token count of
 // each variant needs the most shared memory.
 cudaError_t prepare_decode(const archead_pack *p) {
-  if (!decode_supported(p->d_pad, p->nls, p->g)) return cudaSuccess;
+  if (!decode_supported(p->d_pad, p->nls_dec, p->g)) return cudaSuccess;
   DecodeParams dp = decode_params(p, nullptr, kDecodeWideTokens);
   for (int M : {8, 16, 32, kDecodeWideTokens}) {
-    dp.variant = decode_variant(p->d_pad, p->nls, p->g, M);
+    dp.variant = decode_variant(p->d_pad, p->nls_dec, p->g, M);
     dp.M = std::min(M, variant_tokens(dp.variant));
     const cudaError_t e = launch_decode(dp, 0, nullptr, false);
     if (e != cudaSuccess) return e;

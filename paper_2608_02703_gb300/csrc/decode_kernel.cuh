@@ -465,7 +465,7 @@ __global__ void __launch_bounds__(variant_threads(VAR), 1) decode_kernel(const _
     float a_lo[MT], a_hi[MT];
 #pragma unroll
     for (int mt = 0; mt < MT; ++mt) a_lo[mt] = a_hi[mt] = 1.f;
-    if (kRatio && active && p.nls > p.nls_core) {
+    if (kRatio && active && p.has_corr) {
       const int64_t rb = ((int64_t)TL * unit + tsel) * kTileRows + mi0 * 16 + gq;
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt) {
@@ -701,9 +701,14 @@ __global__ void __launch_bounds__(variant_threads(VAR), 1) decode_kernel(const _
       }
     }
 
-    // Rank-r branches as extra k steps (core: factor 1; correction: row scale
-    // of A_w), with the same copy-then-release of each stage.  Narrow: part
-    // sums again, promoted at the end of each branch.
+    // Rank-r branches as extra k steps, with the same copy-then-release of
+    // each stage.  Columns k < core_cols of the steps are the core's, the
+    // rest the correction's (row scale of A_w).  INT8 format: each step is
+    // one branch's.  SC4 format: the branches lie back to back (the paper's
+    // r_c = 10, r_r = 6 share one step), so a step may hold both: its A
+    // operand is split by masks, the core part goes straight into acc
+    // (factor 1), the correction's into part (narrow, promoted once at the
+    // end) or into acc scaled by 1 / s_a before its first column (wide).
 #pragma unroll
     for (int a = 0; a < (kRatio ? 1 : MT); ++a)
 #pragma unroll
@@ -761,19 +766,11 @@ __global__ void __launch_bounds__(variant_threads(VAR), 1) decode_kernel(const _
       for (int l = 0; l < Geom::kLrSteps; ++l) {
         if (l >= nl) break;
         const int ls = ls0 + l;
-        if (kRatio && ls == p.nls_core) {  // first correction step: continue in units of s_a
-#pragma unroll
-          for (int mt = 0; mt < MT; ++mt) {
-            const float il = __fdividef(1.f, a_lo[mt]), ih = __fdividef(1.f, a_hi[mt]);
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-              acc[mt][nt][0] *= il;
-              acc[mt][nt][1] *= il;
-              acc[mt][nt][2] *= ih;
-              acc[mt][nt][3] *= ih;
-            }
-          }
-        }
+        const int kb = min(max(p.core_cols - 16 * ls, 0), 16);  // k < kb: core columns of this step
+        // Core halves of this lane's k pairs (2cq, 2cq+1) and (2cq+8, 2cq+9).
+        const uint32_t m0 = (2 * cq < kb ? 0x0000FFFFu : 0u) | (2 * cq + 1 < kb ? 0xFFFF0000u : 0u);
+        const uint32_t m1 = (2 * cq + 8 < kb ? 0x0000FFFFu : 0u) | (2 * cq + 9 < kb ? 0xFFFF0000u : 0u);
+        const bool first_corr = kb < 16 && 16 * ls <= p.core_cols;  // the correction starts in this step
         uint32_t bh[NT][2], bl[NT][2];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
@@ -786,33 +783,101 @@ __global__ void __launch_bounds__(variant_threads(VAR), 1) decode_kernel(const _
           bl[nt][0] = l2.x;
           bl[nt][1] = l2.y;
         }
+        if constexpr (!kSC4) {
+          // INT8 format: every step belongs to one branch (core_cols = the
+          // core's padded columns); part sums promoted at each branch's end.
+          const int nls_core = p.core_cols >> 4;
+          if (kRatio && ls == nls_core) {  // first correction step: continue in units of s_a
+#pragma unroll
+            for (int mt = 0; mt < MT; ++mt) {
+              const float il = __fdividef(1.f, a_lo[mt]), ih = __fdividef(1.f, a_hi[mt]);
+#pragma unroll
+              for (int nt = 0; nt < NT; ++nt) {
+                acc[mt][nt][0] *= il;
+                acc[mt][nt][1] *= il;
+                acc[mt][nt][2] *= ih;
+                acc[mt][nt][3] *= ih;
+              }
+            }
+          }
+#pragma unroll
+          for (int mt = 0; mt < MT; ++mt) {
+            uint32_t a[4];
+            unpack_int8x8(lw[l][mt].x, lw[l][mt].y, a);
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+              float (&pt)[4] = kRatio ? acc[mt][nt] : part[kRatio ? 0 : mt][kRatio ? 0 : nt];
+              mma_bf16_16816(pt, a, bh[nt][0], bh[nt][1]);
+              mma_bf16_16816(pt, a, bl[nt][0], bl[nt][1]);
+            }
+          }
+          if constexpr (!kRatio) {
+            if (ls + 1 == nls_core || ls + 1 == p.nls) {
+              const bool corr = ls + 1 == p.nls && p.has_corr;  // the correction ends with the last stage
+#pragma unroll
+              for (int mt = 0; mt < MT; ++mt) {
+                promote<NT>(acc[mt], part[mt], corr ? a_lo[mt] : 1.f, corr ? a_hi[mt] : 1.f);
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                  for (int c = 0; c < 4; ++c) part[mt][nt][c] = 0.f;
+              }
+            }
+          }
+          continue;
+        }
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
           uint32_t a[4];
           unpack_int8x8(lw[l][mt].x, lw[l][mt].y, a);
+          if (kb > 0) {  // core columns
+            uint32_t ac[4] = {a[0], a[1], a[2], a[3]};
+            if (kb < 16) {
+              ac[0] &= m0;
+              ac[1] &= m0;
+              ac[2] &= m1;
+              ac[3] &= m1;
+            }
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
-            float (&pt)[4] = kRatio ? acc[mt][nt] : part[kRatio ? 0 : mt][kRatio ? 0 : nt];
-            mma_bf16_16816(pt, a, bh[nt][0], bh[nt][1]);
-            mma_bf16_16816(pt, a, bl[nt][0], bl[nt][1]);
+            for (int nt = 0; nt < NT; ++nt) {
+              mma_bf16_16816(acc[mt][nt], ac, bh[nt][0], bh[nt][1]);
+              mma_bf16_16816(acc[mt][nt], ac, bl[nt][0], bl[nt][1]);
+            }
           }
-        }
-        if constexpr (!kRatio) {
-          if (ls + 1 == p.nls_core || ls + 1 == p.nls) {
-            const bool corr = ls + 1 == p.nls && p.nls > p.nls_core;  // the correction ends with the last stage
+          if (kb < 16) {  // correction columns
+            if (kb > 0) {
+              a[0] &= ~m0;
+              a[1] &= ~m0;
+              a[2] &= ~m1;
+              a[3] &= ~m1;
+            }
+            if (kRatio && first_corr) {  // continue in units of s_a
+              const float il = __fdividef(1.f, a_lo[mt]), ih = __fdividef(1.f, a_hi[mt]);
 #pragma unroll
-            for (int mt = 0; mt < MT; ++mt) {
-              promote<NT>(acc[mt], part[mt], corr ? a_lo[mt] : 1.f, corr ? a_hi[mt] : 1.f);
+              for (int nt = 0; nt < NT; ++nt) {
+                acc[mt][nt][0] *= il;
+                acc[mt][nt][1] *= il;
+                acc[mt][nt][2] *= ih;
+                acc[mt][nt][3] *= ih;
+              }
+            }
 #pragma unroll
-              for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-                for (int c = 0; c < 4; ++c) part[mt][nt][c] = 0.f;
+            for (int nt = 0; nt < NT; ++nt) {
+              float (&pt)[4] = kRatio ? acc[mt][nt] : part[kRatio ? 0 : mt][kRatio ? 0 : nt];
+              mma_bf16_16816(pt, a, bh[nt][0], bh[nt][1]);
+              mma_bf16_16816(pt, a, bl[nt][0], bl[nt][1]);
             }
           }
         }
       }
     }
-    if (kRatio && active && p.nls > p.nls_core) {  // the correction's row scale
+    if constexpr (!kRatio && kSC4) {  // the correction's row scale
+      if (active && p.has_corr) {
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) promote<NT>(acc[mt], part[mt], a_lo[mt], a_hi[mt]);
+      }
+    }
+    if (kRatio && active && p.has_corr) {  // the correction's row scale
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt)
 #pragma unroll

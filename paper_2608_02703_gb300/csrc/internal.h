@@ -65,7 +65,10 @@ struct DecodeParams {
   const uint16_t *x;    // hidden states [M_total][d] bf16 (this chunk starts at row m0)
   const uint32_t *ts;   // t hi/lo fragments for this token chunk
   int64_t V;
-  int num_tiles, d, d_pad, G_pad, g, nls, nls_core;
+  int num_tiles, d, d_pad, G_pad, g;
+  int nls;              // 16-wide rank-r steps of lr_codes (decode layout)
+  int core_cols;        // rank-r columns before the correction's: k < core_cols of the steps are A_c
+  int has_corr;         // r_r > 0
   int sc4, G_pad2;      // SC4 format flag; byte rows of scale codes per tile
   int M;                // tokens in this chunk (1..16)
   int m0;               // index of the chunk's first token
@@ -93,6 +96,8 @@ struct PrepassParams {
   float *partial;          // per-split partial sums (workspace)
   int *counters;           // one per (columns, tokens) block pair, zero between calls
   uint32_t *ts;            // decode t fragments, per 16-token chunk
+  int ts_nls, ts_core;     // their steps and core columns (the decode layout of the rank-r codes)
+  int ts_compact;          // decode layout packs core and correction back to back
   uint16_t *T;             // prefill extended-K operand [M][2*LR] bf16 (may be NULL)
 };
 
@@ -110,6 +115,11 @@ struct archead_pack {
   int sm_count = 0;
   int64_t V = 0, V_pad = 0;
   int d = 0, rc = 0, rr = 0, g = 0, G = 0, rcp = 0, rrp = 0, lr = 0, nls = 0, nls_core = 0;
+  // Decode layout of the rank-r codes: core and correction columns back to
+  // back, padded once to 16 (lr_codes_dec; the same buffer as lr_codes when
+  // that saves no step, with core_cols = rcp).
+  int nls_dec = 0, core_cols = 0;
+  uint8_t *lr_codes_dec = nullptr;
   int d_pad = 0, G_pad = 0;  // d rounded up to 128, and its group count
   int num_tiles = 0;
   int sc4 = 0;               // ARCHEAD_FORMAT_SC4

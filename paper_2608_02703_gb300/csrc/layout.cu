@@ -152,6 +152,11 @@ cudaError_t launch_build_layouts(archead_pack *p, const uint8_t *res_codes, cons
   if (p->nls > 0)
     build_lr_codes_kernel<<<p->num_tiles * p->nls, 256, 0, s>>>(core_u, corr_a, corr_a_scale, p->lr_codes, p->V, p->rc,
                                                                  p->rr, p->rcp, p->nls, p->sc4);
+  // The decode layout, when it differs: the same codes with the core's
+  // columns unpadded (rcp taken as r_c) and nls_dec steps.
+  if (p->nls_dec > 0 && p->lr_codes_dec != p->lr_codes)
+    build_lr_codes_kernel<<<p->num_tiles * p->nls_dec, 256, 0, s>>>(core_u, corr_a, corr_a_scale, p->lr_codes_dec, p->V,
+                                                                     p->rc, p->rr, p->rc, p->nls_dec, p->sc4);
   build_row_scales_kernel<<<256, 256, 0, s>>>(p->rr > 0 ? corr_a_scale : nullptr, p->s_a, p->V, p->V_pad);
   if (p->lr > 0)
     build_lr_t_kernel<<<256, 256, 0, s>>>(p->q_v, p->q_b, p->lr_t, p->d, p->d_pad, p->rc, p->rr, p->rcp, p->lr);

@@ -72,14 +72,14 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
     set_last_error_message("archead_forward_decode_noalloc: M must be at most 16");
     return ARCHEAD_ERR_UNSUPPORTED;
   }
-  if (!decode_supported(pack->d_pad, pack->nls, pack->g)) {
+  if (!decode_supported(pack->d_pad, pack->nls_dec, pack->g)) {
     set_last_error_message("archead_forward_decode_noalloc: the decode kernel does not support this head shape");
     return ARCHEAD_ERR_UNSUPPORTED;
   }
   // Scratch: [block counters | pre-pass partial sums | rank-r fragments of one 16-token chunk].
   const int pairs = prepass_pairs((int)M, pack->lr);
   const size_t partial_bytes = (prepass_partial_bytes((int)M, pack->lr, pack->d) + 255) / 256 * 256;
-  const size_t ts_bytes = (size_t)(pack->nls > 0 ? pack->nls : 1) * 1024;
+  const size_t ts_bytes = (size_t)(pack->nls_dec > 0 ? pack->nls_dec : 1) * 1024;
   const size_t need = kNoallocCounterBytes + partial_bytes + ts_bytes;
   if (need > kNoallocScratchBytes || (size_t)pairs * sizeof(int) > kNoallocCounterBytes) {
     set_last_error_message(
@@ -117,7 +117,7 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
   dp.ts = ts;
   dp.M = (int)M;
   dp.m0 = 0;
-  dp.variant = decode_variant(pack->d_pad, pack->nls, pack->g, (int)M);
+  dp.variant = decode_variant(pack->d_pad, pack->nls_dec, pack->g, (int)M);
   dp.out = logits;
   dp.out_fp32 = out_dtype == ARCHEAD_OUT_FP32;
   const int units = decode_num_units(pack, dp.variant);

@@ -111,7 +111,6 @@ __global__ void __launch_bounds__(256) prepass_kernel(PrepassParams p) {
   if (!last_block) return;
   __threadfence();
 
-  const int nls = p.lr / 16;
   for (int e = threadIdx.x; e < kPreTok * kPreCols; e += blockDim.x) {
     const int m = e / kPreCols, c = e % kPreCols;
     // Tokens past M in this 16-token chunk get zero fragments.
@@ -151,15 +150,20 @@ __global__ void __launch_bounds__(256) prepass_kernel(PrepassParams p) {
         row[2 * p.rcp + p.rrp + jj] = lo;
       }
     }
-    if (p.ts) {
+    // Column of the decode layout: the same as kk, or with core and
+    // correction back to back (core columns as they are, correction ones
+    // after the r_c core ones, and the core's padding columns, whose t is
+    // zero, moved past the correction to zero the rest of the last step).
+    const int pos = !p.ts_compact ? kk : kk < p.rc ? kk : kk < p.rcp ? kk + p.rr : p.ts_core + (kk - p.rcp);
+    if (p.ts && pos < 16 * p.ts_nls) {
       // B-fragment of step ls: register (k16 >= 8), lane = 4*(token%8) + (k16%8)/2.
       const int chunk = mg / kDecodeMaxTokens, nl = mg % kDecodeMaxTokens;
       const int nt = nl >> 3, gq = nl & 7;
-      const int ls = kk >> 4, k16 = kk & 15;
+      const int ls = pos >> 4, k16 = pos & 15;
       const int reg = k16 >> 3, cq = (k16 & 7) >> 1, h = k16 & 1;
       const int ln = gq * 4 + cq;
       uint16_t *ts16 = reinterpret_cast<uint16_t *>(p.ts);
-      const int64_t base = ((((int64_t)chunk * nls + ls) * 2) * 2 + nt) * 32 + ln;  // hl = 0
+      const int64_t base = ((((int64_t)chunk * p.ts_nls + ls) * 2) * 2 + nt) * 32 + ln;  // hl = 0
       ts16[base * 4 + reg * 2 + h] = hi;
       ts16[(base + 2 * 32) * 4 + reg * 2 + h] = lo;  // hl = 1
     }
