@@ -124,7 +124,7 @@ struct ForwardPlan {
 ForwardPlan plan_decode(archead_pack *p, int64_t M, bool ce) {
   ForwardPlan f;
   Carve c;
-  f.variant = decode_variant(p->d_pad, p->nls_dec, p->g, (int)std::min<int64_t>(M, kDecodeWideTokens));
+  f.variant = decode_variant(p, (int)std::min<int64_t>(M, kDecodeWideTokens));
   f.chunk_tokens = decode_variant_tokens(f.variant);
   f.nchunks = (int)((M + f.chunk_tokens - 1) / f.chunk_tokens);
   f.partial_off = c.take(prepass_partial_bytes((int)M, p->lr, p->d));
@@ -263,7 +263,7 @@ archead_status run_forward(archead_pack *p, const void *x, int64_t M, void *out,
   // kernel under AUTO.
   bool decode = path == ARCHEAD_PATH_DECODE;
   if (path == ARCHEAD_PATH_AUTO && M <= kDecodeWideTokens && decode_supported(p->d_pad, p->nls_dec, p->g)) {
-    const int tok = decode_variant_tokens(decode_variant(p->d_pad, p->nls_dec, p->g, (int)M));
+    const int tok = decode_variant_tokens(decode_variant(p, (int)M));
     decode = (M + tok - 1) / tok <= 3;
   }
   if (decode) return run_decode(p, x, M, out, out_fp32, targets, ce, amax_idx, amax_val, row0, parts3, s);

@@ -30,12 +30,31 @@ static bool wide_fits(int d_pad, int nls, int g, int variant) {
   return decode_plan(d_pad, nls, g, variant_tokens(variant), variant).stages >= 4;
 }
 
-int decode_variant(int d_pad, int nls, int g, int M) {
+// Resident x in units of two tiles: for the paper's format (measured faster
+// there: 63.8 against 65.7 us at M = 1 on the Qwen3-8B head), and for INT8
+// heads whose four-tile units fill the last round of blocks at least 5 %
+// worse than two-tile units would (Gemma-shaped head: 78.9 against 80.0 us;
+// on the Qwen3-8B head, where both fill it alike, two-tile units are 2.7 %
+// slower).
+static bool half_units(const archead_pack *p) {
+  if (p->d_pad % (stage_chunks(kDecResidentH) * kChunkK) != 0) return false;  // whole stages of four chunks
+  if (p->sc4) return true;
+  const auto fill = [&](int tiles_per_unit) {
+    const int units = (p->num_tiles + tiles_per_unit - 1) / tiles_per_unit;
+    const int rounds = (units + p->sm_count - 1) / p->sm_count;
+    return (double)units / ((double)rounds * p->sm_count);
+  };
+  return fill(2) > fill(4) + 0.05;
+}
+
+int decode_variant(const archead_pack *p, int M) {
+  const int d_pad = p->d_pad, nls = p->nls_dec, g = p->g;
   if (M > 32 && wide_fits(d_pad, nls, g, kDecWide8)) return kDecWide8;
   if (M > 16 && wide_fits(d_pad, nls, g, kDecWide4)) return kDecWide4;
   if (M > 8) return kDecStreamed2;
-  const DecodePlan pl = decode_plan(d_pad, nls, g, M, kDecResident1);
-  return pl.stages >= 2 && pl.xs_off >= (size_t)96 * 1024 ? kDecResident1 : kDecStreamed2;
+  const int resident = half_units(p) ? kDecResidentH : kDecResident1;
+  const DecodePlan pl = decode_plan(d_pad, nls, g, M, resident);
+  return pl.stages >= 2 && pl.xs_off >= (size_t)96 * 1024 ? resident : kDecStreamed2;
 }
 
 extern template cudaError_t launch_decode_fmt<true>(const DecodeParams &, int, cudaStream_t, bool);
@@ -51,7 +70,7 @@ cudaError_t prepare_decode(const archead_pack *p) {
   if (!decode_supported(p->d_pad, p->nls_dec, p->g)) return cudaSuccess;
   DecodeParams dp = decode_params(p, nullptr, kDecodeWideTokens);
   for (int M : {8, 16, 32, kDecodeWideTokens}) {
-    dp.variant = decode_variant(p->d_pad, p->nls_dec, p->g, M);
+    dp.variant = decode_variant(p, M);
     dp.M = std::min(M, variant_tokens(dp.variant));
     const cudaError_t e = launch_decode(dp, 0, nullptr, false);
     if (e != cudaSuccess) return e;

@@ -41,7 +41,10 @@ constexpr int kSmemLimit = 227 * 1024;
 // Kernel instances ("variants"), chosen per launch from the token count and
 // the head's width:
 //  - kDecResident1: up to 8 tokens (one 8-token n-tile), hidden states staged
-//    once in shared memory as fp16;
+//    once in shared memory as fp16; kDecResidentH the same in units of two
+//    tiles (eight warps of two m-tiles, four 64-wide chunks per stage), for
+//    the paper's format and for heads whose four-tile units leave the last
+//    round of blocks poorly filled;
 //  - kDecStreamed2: 9..16 tokens (two n-tiles), and up to 8 tokens of heads
 //    so wide that x of 8 tokens does not fit next to a working ring.  The
 //    hidden states are not kept in shared memory (16 rows of d would take
@@ -70,27 +73,27 @@ constexpr int kSmemLimit = 227 * 1024;
 //    group-scale units (145-152 us for 17-32 tokens, no better; 207 us with
 //    the paper's format, which spilled), and kDecWide8 with sixteen warps of
 //    two m-tiles and four n-tiles each (265-278 us).
-enum DecodeVariant { kDecResident1 = 0, kDecStreamed2 = 1, kDecWide4 = 2, kDecWide8 = 3 };
+enum DecodeVariant { kDecResident1 = 0, kDecStreamed2 = 1, kDecWide4 = 2, kDecWide8 = 3, kDecResidentH = 4 };
 
 __host__ __device__ constexpr int variant_nt(int v) {  // 8-token n-tiles
-  return v == kDecResident1 ? 1 : v == kDecStreamed2 ? 2 : v == kDecWide4 ? 4 : 8;
+  return v == kDecResident1 || v == kDecResidentH ? 1 : v == kDecStreamed2 ? 2 : v == kDecWide4 ? 4 : 8;
 }
 __host__ __device__ constexpr int variant_cw(int v) {  // consumer warps
-  return v == kDecResident1 || v == kDecWide8 ? 8 : 16;
+  return v == kDecStreamed2 || v == kDecWide4 ? 16 : 8;
 }
 __host__ __device__ constexpr int variant_mt(int v) {  // 16-row m-tiles per consumer warp
-  return v == kDecResident1 ? 4 : v == kDecWide4 ? 1 : 2;
+  return v == kDecResident1 ? 4 : v == kDecWide4 ? 1 : 2;  // kDecResidentH: 2
 }
 // 128-row tiles per unit: the consumer warps cover them, MT m-tiles each.
 __host__ __device__ constexpr int variant_tiles(int v) { return variant_cw(v) * variant_mt(v) / 8; }
 __host__ __device__ constexpr int variant_threads(int v) { return (variant_cw(v) + 1) * 32; }  // + producer warp
 __host__ __device__ constexpr int variant_tokens(int v) { return 8 * variant_nt(v); }  // largest M of one launch
-__host__ __device__ constexpr bool streams_x(int v) { return v != kDecResident1; }
+__host__ __device__ constexpr bool streams_x(int v) { return v != kDecResident1 && v != kDecResidentH; }
 // Token stride of the per-group sums of x (at least 16: the smallest instances' layout).
 __host__ __device__ constexpr int xsum_tokens(int v) { return variant_tokens(v) < 16 ? 16 : variant_tokens(v); }
 // 64-wide chunks of d per ring stage.  The shared-memory plan and the kernel
 // instance launched both take it from here.
-__host__ __device__ constexpr int stage_chunks(int v) { return 2; }
+__host__ __device__ constexpr int stage_chunks(int v) { return v == kDecResidentH ? 4 : 2; }
 // One chunk of x in a stage: the instance's tokens x 64 of d, bf16, 128-byte swizzle.
 __host__ __device__ constexpr int x_chunk_bytes(int v) { return variant_tokens(v) < 16 ? 16 * kChunkK * 2 : variant_tokens(v) * kChunkK * 2; }
 
@@ -125,7 +128,8 @@ static DecodePlan decode_plan(int d_pad, int nls, int g, int M, int variant) {
   const size_t stage_bytes = variant == kDecResident1   ? GeomOf<kDecResident1>::kBytes
                              : variant == kDecStreamed2 ? GeomOf<kDecStreamed2>::kBytes
                              : variant == kDecWide4     ? GeomOf<kDecWide4>::kBytes
-                                                        : GeomOf<kDecWide8>::kBytes;
+                             : variant == kDecWide8     ? GeomOf<kDecWide8>::kBytes
+                                                        : GeomOf<kDecResidentH>::kBytes;
   const size_t xs_bytes = xs ? 0 : (size_t)M * xs_row_elems(d_pad) * 2;
   // rank-r fragments of the 16-token chunks the launch covers
   const size_t ts_bytes = (size_t)((variant_tokens(variant) + kDecodeMaxTokens - 1) / kDecodeMaxTokens) * nls * 1024;
@@ -1018,8 +1022,10 @@ template <bool kSC4>
 cudaError_t launch_decode_fmt(const DecodeParams &dp, int grid, cudaStream_t s, bool pdl) {
   const DecodePlan pl = decode_plan(dp.d_pad, dp.nls, dp.g, dp.M, dp.variant);
   if (pl.stages < 2 || pl.sc != stage_chunks(dp.variant)) return cudaErrorInvalidValue;
+  if (dp.d_pad % (pl.sc * kChunkK) != 0) return cudaErrorInvalidValue;  // the residual in whole stages
   if (dp.M < 1 || dp.M > variant_tokens(dp.variant)) return cudaErrorInvalidValue;
   if (dp.variant == kDecResident1) return launch_g<kDecResident1, kSC4>(dp, grid, s, pl, pdl);
+  if (dp.variant == kDecResidentH) return launch_g<kDecResidentH, kSC4>(dp, grid, s, pl, pdl);
   if (dp.variant < kDecStreamed2 || dp.variant > kDecWide8) return cudaErrorInvalidValue;
   DecodeParams dx = dp;
   if (grid > 0 && !make_tma_map_bf16(&dx.tmap_x, dp.x, dp.M_total, dp.d, variant_tokens(dp.variant)))

@@ -117,7 +117,7 @@ extern "C" ARCHEAD_API archead_status archead_forward_decode_noalloc(archead_pac
   dp.ts = ts;
   dp.M = (int)M;
   dp.m0 = 0;
-  dp.variant = decode_variant(pack->d_pad, pack->nls_dec, pack->g, (int)M);
+  dp.variant = decode_variant(pack, (int)M);
   dp.out = logits;
   dp.out_fp32 = out_dtype == ARCHEAD_OUT_FP32;
   const int units = decode_num_units(pack, dp.variant);
