@@ -51,10 +51,16 @@ int decode_variant(const archead_pack *p, int M) {
   const int d_pad = p->d_pad, nls = p->nls_dec, g = p->g;
   if (M > 32 && wide_fits(d_pad, nls, g, kDecWide8)) return kDecWide8;
   if (M > 16 && wide_fits(d_pad, nls, g, kDecWide4)) return kDecWide4;
-  if (M > 8) return kDecStreamed2;
+  // Streamed x, two n-tiles: in two-tile units where d is whole four-chunk
+  // stages and that ring keeps at least four stages.
+  const int streamed =
+      d_pad % (stage_chunks(kDecStreamedH) * kChunkK) == 0 && wide_fits(d_pad, nls, g, kDecStreamedH)
+          ? kDecStreamedH
+          : kDecStreamed2;
+  if (M > 8) return streamed;
   const int resident = half_units(p) ? kDecResidentH : kDecResident1;
   const DecodePlan pl = decode_plan(d_pad, nls, g, M, resident);
-  return pl.stages >= 2 && pl.xs_off >= (size_t)96 * 1024 ? resident : kDecStreamed2;
+  return pl.stages >= 2 && pl.xs_off >= (size_t)96 * 1024 ? resident : streamed;
 }
 
 extern template cudaError_t launch_decode_fmt<true>(const DecodeParams &, int, cudaStream_t, bool);

@@ -56,6 +56,11 @@ constexpr int kSmemLimit = 227 * 1024;
 //    there with two n-tiles).  Sixteen consumer warps of two m-tiles each
 //    (92.1 us at M = 16 against 94.2 with eight warps of four; for M <= 8 the
 //    resident instance keeps eight warps: 67.7 against 73.8 us with sixteen).
+//    kDecStreamedH the same in units of two tiles (sixteen warps of one
+//    m-tile, four 64-wide chunks per stage), where d is whole stages of four
+//    chunks: 89.5 against 92.1 us at M = 16 on the Qwen3-8B-shaped head,
+//    100.5 against 110.7 on the Gemma-shaped one.  (The 32-token instance
+//    with four-chunk stages was slower: 174 against 154 us.)
 // Measured alternatives that were slower on the Qwen3-8B-shaped head (and not
 // kept): 16 tokens of x resident as fp16 with a 2-chunk ring (98.4 us at
 // M = 16 against 94.8) or a 1-chunk ring with the next stage prefetched into
@@ -73,16 +78,18 @@ constexpr int kSmemLimit = 227 * 1024;
 //    group-scale units (145-152 us for 17-32 tokens, no better; 207 us with
 //    the paper's format, which spilled), and kDecWide8 with sixteen warps of
 //    two m-tiles and four n-tiles each (265-278 us).
-enum DecodeVariant { kDecResident1 = 0, kDecStreamed2 = 1, kDecWide4 = 2, kDecWide8 = 3, kDecResidentH = 4 };
+enum DecodeVariant {
+  kDecResident1 = 0, kDecStreamed2 = 1, kDecWide4 = 2, kDecWide8 = 3, kDecResidentH = 4, kDecStreamedH = 5
+};
 
 __host__ __device__ constexpr int variant_nt(int v) {  // 8-token n-tiles
-  return v == kDecResident1 || v == kDecResidentH ? 1 : v == kDecStreamed2 ? 2 : v == kDecWide4 ? 4 : 8;
+  return v == kDecResident1 || v == kDecResidentH ? 1 : v == kDecStreamed2 || v == kDecStreamedH ? 2 : v == kDecWide4 ? 4 : 8;
 }
 __host__ __device__ constexpr int variant_cw(int v) {  // consumer warps
-  return v == kDecStreamed2 || v == kDecWide4 ? 16 : 8;
+  return v == kDecStreamed2 || v == kDecStreamedH || v == kDecWide4 ? 16 : 8;
 }
 __host__ __device__ constexpr int variant_mt(int v) {  // 16-row m-tiles per consumer warp
-  return v == kDecResident1 ? 4 : v == kDecWide4 ? 1 : 2;  // kDecResidentH: 2
+  return v == kDecResident1 ? 4 : v == kDecWide4 || v == kDecStreamedH ? 1 : 2;  // kDecResidentH: 2
 }
 // 128-row tiles per unit: the consumer warps cover them, MT m-tiles each.
 __host__ __device__ constexpr int variant_tiles(int v) { return variant_cw(v) * variant_mt(v) / 8; }
@@ -93,7 +100,7 @@ __host__ __device__ constexpr bool streams_x(int v) { return v != kDecResident1 
 __host__ __device__ constexpr int xsum_tokens(int v) { return variant_tokens(v) < 16 ? 16 : variant_tokens(v); }
 // 64-wide chunks of d per ring stage.  The shared-memory plan and the kernel
 // instance launched both take it from here.
-__host__ __device__ constexpr int stage_chunks(int v) { return v == kDecResidentH ? 4 : 2; }
+__host__ __device__ constexpr int stage_chunks(int v) { return v == kDecResidentH || v == kDecStreamedH ? 4 : 2; }
 // One chunk of x in a stage: the instance's tokens x 64 of d, bf16, 128-byte swizzle.
 __host__ __device__ constexpr int x_chunk_bytes(int v) { return variant_tokens(v) < 16 ? 16 * kChunkK * 2 : variant_tokens(v) * kChunkK * 2; }
 
@@ -129,7 +136,8 @@ static DecodePlan decode_plan(int d_pad, int nls, int g, int M, int variant) {
                              : variant == kDecStreamed2 ? GeomOf<kDecStreamed2>::kBytes
                              : variant == kDecWide4     ? GeomOf<kDecWide4>::kBytes
                              : variant == kDecWide8     ? GeomOf<kDecWide8>::kBytes
-                                                        : GeomOf<kDecResidentH>::kBytes;
+                             : variant == kDecResidentH ? GeomOf<kDecResidentH>::kBytes
+                                                        : GeomOf<kDecStreamedH>::kBytes;
   const size_t xs_bytes = xs ? 0 : (size_t)M * xs_row_elems(d_pad) * 2;
   // rank-r fragments of the 16-token chunks the launch covers
   const size_t ts_bytes = (size_t)((variant_tokens(variant) + kDecodeMaxTokens - 1) / kDecodeMaxTokens) * nls * 1024;
@@ -1026,11 +1034,13 @@ cudaError_t launch_decode_fmt(const DecodeParams &dp, int grid, cudaStream_t s, 
   if (dp.M < 1 || dp.M > variant_tokens(dp.variant)) return cudaErrorInvalidValue;
   if (dp.variant == kDecResident1) return launch_g<kDecResident1, kSC4>(dp, grid, s, pl, pdl);
   if (dp.variant == kDecResidentH) return launch_g<kDecResidentH, kSC4>(dp, grid, s, pl, pdl);
-  if (dp.variant < kDecStreamed2 || dp.variant > kDecWide8) return cudaErrorInvalidValue;
+  if (dp.variant != kDecStreamed2 && dp.variant != kDecStreamedH && dp.variant != kDecWide4 && dp.variant != kDecWide8)
+    return cudaErrorInvalidValue;
   DecodeParams dx = dp;
   if (grid > 0 && !make_tma_map_bf16(&dx.tmap_x, dp.x, dp.M_total, dp.d, variant_tokens(dp.variant)))
     return cudaErrorInvalidValue;
   if (dp.variant == kDecStreamed2) return launch_g<kDecStreamed2, kSC4>(dx, grid, s, pl, pdl);
+  if (dp.variant == kDecStreamedH) return launch_g<kDecStreamedH, kSC4>(dx, grid, s, pl, pdl);
   if (dp.variant == kDecWide4) return launch_g<kDecWide4, kSC4>(dx, grid, s, pl, pdl);
   return launch_g<kDecWide8, kSC4>(dx, grid, s, pl, pdl);
 }

@@ -187,7 +187,8 @@ int decode_parts_per_unit(int variant);  // cross-entropy partial blocks per uni
 bool decode_supported(int d_pad, int nls, int g);
 // Kernel instance for a launch of M tokens (M > 64: the instance every
 // 64-token chunk runs): 0 (4: units of two tiles) one 8-token n-tile, x
-// resident; 1, 2, 3 two, four and eight n-tiles, x streamed.
+// resident; 1 (5: units of two tiles), 2, 3 two, four and eight n-tiles, x
+// streamed.
 int decode_variant(const archead_pack *p, int M);
 cudaError_t launch_prefill(const archead_pack *pk, const void *x, int M, const uint16_t *T, void *out, int out_fp32,
                            bool argmax, const int32_t *targets, int row0, float2 *ce_part, float *ce_tlogit,
