@@ -131,7 +131,7 @@ ForwardPlan plan_decode(archead_pack *p, int64_t M, bool ce) {
   // rank-r fragments, in 16-token chunks
   f.ts_off = c.take((size_t)((M + kDecodeMaxTokens - 1) / kDecodeMaxTokens) * std::max(p->nls_dec, 1) * 1024);
   if (ce) {
-    f.ce_part_off = c.take((size_t)decode_num_units(p, f.variant) * decode_parts_per_unit(f.variant) * M * sizeof(float2));
+    f.ce_part_off = c.take((size_t)decode_num_units(p, f.variant) * decode_parts_per_unit(f.variant, p->sc4) * M * sizeof(float2));
     f.tlogit_off = c.take((size_t)M * sizeof(float));
   }
   f.total = c.off;
@@ -195,7 +195,7 @@ archead_status run_decode(archead_pack *p, const void *x, int64_t M, void *out, 
   if (ce_mode) {
     cudaEvent_t ev = nullptr;
     timer_begin(p, "ce_finalize", s, &ev);
-    const int parts = units * decode_parts_per_unit(f.variant);
+    const int parts = units * decode_parts_per_unit(f.variant, p->sc4);
     cudaError_t e =
         greedy   ? launch_argmax_finalize(dp.ce_part, parts, (int)M, amax_idx, amax_val, s)
         : parts3 ? launch_lse_partial_finalize(dp.ce_part, parts, dp.ce_tlogit, targets, row0, p->V, (int)M, parts3, s)

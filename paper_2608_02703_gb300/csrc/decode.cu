@@ -12,7 +12,7 @@ int decode_num_units(const archead_pack *p, int variant) {
 
 int decode_variant_tokens(int variant) { return variant_tokens(variant); }
 
-int decode_parts_per_unit(int variant) { return variant_cw(variant); }
+int decode_parts_per_unit(int variant, bool sc4) { return variant_cw(variant, sc4); }
 
 bool decode_supported(int d_pad, int nls, int g) {
   return decode_plan(d_pad, nls, g, kDecodeMaxTokens, kDecStreamed2).stages >= 2;
@@ -33,9 +33,9 @@ static bool wide_fits(int d_pad, int nls, int g, int variant) {
 // Resident x in units of two tiles: for the paper's format (measured faster
 // there: 63.8 against 65.7 us at M = 1 on the Qwen3-8B head), and for INT8
 // heads whose four-tile units fill the last round of blocks at least 5 %
-// worse than two-tile units would (Gemma-shaped head: 78.9 against 80.0 us;
-// on the Qwen3-8B head, where both fill it alike, two-tile units are 2.7 %
-// slower).
+// worse than two-tile units would (Gemma-shaped head: 77.4 against 79.3 us
+// with sixteen warps of one m-tile; on the Qwen3-8B head, where both fill it
+// alike, two-tile units are 2.7 % slower).
 static bool half_units(const archead_pack *p) {
   if (p->d_pad % (stage_chunks(kDecResidentH) * kChunkK) != 0) return false;  // whole stages of four chunks
   if (p->sc4) return true;

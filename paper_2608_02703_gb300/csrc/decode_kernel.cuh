@@ -85,15 +85,18 @@ enum DecodeVariant {
 __host__ __device__ constexpr int variant_nt(int v) {  // 8-token n-tiles
   return v == kDecResident1 || v == kDecResidentH ? 1 : v == kDecStreamed2 || v == kDecStreamedH ? 2 : v == kDecWide4 ? 4 : 8;
 }
-__host__ __device__ constexpr int variant_cw(int v) {  // consumer warps
-  return v == kDecStreamed2 || v == kDecStreamedH || v == kDecWide4 ? 16 : 8;
+// Consumer warps and m-tiles per warp; kDecResidentH runs sixteen warps of
+// one m-tile for the INT8 format (Gemma-shaped head: 77.4 against 79.3 us at
+// M = 1) and eight of two for the paper's format (64.1 against 68.0 us).
+__host__ __device__ constexpr int variant_cw(int v, bool sc4 = false) {
+  return v == kDecStreamed2 || v == kDecStreamedH || v == kDecWide4 || (v == kDecResidentH && !sc4) ? 16 : 8;
 }
-__host__ __device__ constexpr int variant_mt(int v) {  // 16-row m-tiles per consumer warp
-  return v == kDecResident1 ? 4 : v == kDecWide4 || v == kDecStreamedH ? 1 : 2;  // kDecResidentH: 2
+__host__ __device__ constexpr int variant_mt(int v, bool sc4 = false) {  // 16-row m-tiles per consumer warp
+  return v == kDecResident1 ? 4 : v == kDecWide4 || v == kDecStreamedH || (v == kDecResidentH && !sc4) ? 1 : 2;
 }
 // 128-row tiles per unit: the consumer warps cover them, MT m-tiles each.
 __host__ __device__ constexpr int variant_tiles(int v) { return variant_cw(v) * variant_mt(v) / 8; }
-__host__ __device__ constexpr int variant_threads(int v) { return (variant_cw(v) + 1) * 32; }  // + producer warp
+__host__ __device__ constexpr int variant_threads(int v, bool sc4) { return (variant_cw(v, sc4) + 1) * 32; }  // + producer
 __host__ __device__ constexpr int variant_tokens(int v) { return 8 * variant_nt(v); }  // largest M of one launch
 __host__ __device__ constexpr bool streams_x(int v) { return v != kDecResident1 && v != kDecResidentH; }
 // Token stride of the per-group sums of x (at least 16: the smallest instances' layout).
@@ -199,13 +202,15 @@ __device__ __forceinline__ float scale_mult_16th(uint32_t b, int sh) {
 // VAR: DecodeVariant (n-tiles of 8 tokens, resident or streamed x); SC:
 // 64-wide chunks per stage; GS: 16-wide k steps per group.
 template <int VAR, int SC, int GS, bool kSC4>
-__global__ void __launch_bounds__(variant_threads(VAR), 1) decode_kernel(const __grid_constant__ DecodeParams p, int stages,
+__global__ void __launch_bounds__(variant_threads(VAR, kSC4), 1) decode_kernel(const __grid_constant__ DecodeParams p, int stages,
                                                                 int xs_off, int ts_off, int xsum_off, int bar_off) {
-  constexpr int kDecWarps = variant_cw(VAR);  // consumer warps
+  constexpr int kDecWarps = variant_cw(VAR, kSC4);  // consumer warps
   constexpr int NT = variant_nt(VAR);          // n-tiles per warp
   constexpr bool kStreamX = streams_x(VAR);
   constexpr bool kF16 = !kStreamX;  // fp16 operands with x staged in shared memory
-  constexpr int MT = variant_mt(VAR);        // m-tiles per consumer warp
+  constexpr int MT = variant_mt(VAR, kSC4);  // m-tiles per consumer warp
+  static_assert(variant_cw(VAR, kSC4) * variant_mt(VAR, kSC4) == variant_cw(VAR) * variant_mt(VAR),
+                "the unit size must not depend on the format");
   constexpr int TL = variant_tiles(VAR);     // 128-row tiles per unit
   constexpr int XT = xsum_tokens(VAR);       // token stride of the per-group sums
   constexpr int XCB = x_chunk_bytes(VAR);    // one chunk of streamed x
@@ -999,7 +1004,7 @@ static cudaError_t launch_t(const DecodeParams &dp, int grid, cudaStream_t s, co
   if (e != cudaSuccess || grid == 0) return e;  // grid 0: opt-in only (prepare_decode)
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(variant_threads(VAR));
+  cfg.blockDim = dim3(variant_threads(VAR, kSC4));
   cfg.dynamicSmemBytes = pl.total;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];

@@ -183,7 +183,7 @@ cudaError_t prepare_decode(const archead_pack *p);
 bool make_tma_map_bf16(CUtensorMap *map, const void *base, int64_t rows, int64_t cols, int box_rows);
 int decode_num_units(const archead_pack *p, int variant);  // units (and ce partial blocks) of a variant
 int decode_variant_tokens(int variant);                    // tokens one launch of a variant takes
-int decode_parts_per_unit(int variant);  // cross-entropy partial blocks per unit and token
+int decode_parts_per_unit(int variant, bool sc4);  // cross-entropy partial blocks per unit and token
 bool decode_supported(int d_pad, int nls, int g);
 // Kernel instance for a launch of M tokens (M > 64: the instance every
 // 64-token chunk runs): 0 (4: units of two tiles) one 8-token n-tile, x
