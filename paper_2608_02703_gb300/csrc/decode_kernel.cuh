@@ -42,9 +42,10 @@ constexpr int kSmemLimit = 227 * 1024;
 // the head's width:
 //  - kDecResident1: up to 8 tokens (one 8-token n-tile), hidden states staged
 //    once in shared memory as fp16; kDecResidentH the same in units of two
-//    tiles (eight warps of two m-tiles, four 64-wide chunks per stage), for
-//    the paper's format and for heads whose four-tile units leave the last
-//    round of blocks poorly filled;
+//    tiles with four 64-wide chunks per stage (eight warps of two m-tiles in
+//    the paper's format, sixteen of one in the INT8 format), for the paper's
+//    format and for heads whose four-tile units leave the last round of
+//    blocks poorly filled;
 //  - kDecStreamed2: 9..16 tokens (two n-tiles), and up to 8 tokens of heads
 //    so wide that x of 8 tokens does not fit next to a working ring.  The
 //    hidden states are not kept in shared memory (16 rows of d would take
