@@ -48,8 +48,12 @@ def test_flat_keys_repeat_the_nested_headline_figures():
                 "prefill": {"M": 4096, "logits": {"ms_per_call": 3.9, "frac_bf16_peak": 0.69}}},
         "gemma": {"decode_sweep": [], "prefill": {"M": 2048, "ce": {"ms_per_call": 3.0, "frac_bf16_peak": 0.51}}},
         "tiny": {"us_per_call": 9.5, "oracle": {"us_per_call": 12000.0}},
+        "crossover": {"rows": [{"M": 16, "auto_us": 89.0, "dense_bf16_us": 204.0},
+                               {"M": 64, "auto_us": 245.4, "dense_bf16_us": 210.7}]},
     }
     flat = bench.flat_keys(res)
+    assert flat["qwen_crossover_m64_auto_us"] == 245.4 and flat["qwen_crossover_m64_dense_bf16_us"] == 210.7
+    assert "qwen_crossover_m16_auto_us" not in flat  # only the rows the headline table quotes
     assert flat["qwen_prefill_m4096_logits_ms"] == 4.2 and flat["qwen_prefill_m4096_ce_frac_bf16_peak"] == 0.58
     assert flat["qwen_decode_m16_us"] == 80.0 and flat["qwen_decode_m1_kernel_frac_hbm"] == 0.77
     assert flat["qwen_sc4_decode_m1_us"] == 66.0 and flat["qwen_sc4_prefill_m4096_logits_ms"] == 3.9
