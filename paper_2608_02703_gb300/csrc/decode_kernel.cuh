@@ -15,20 +15,22 @@
 // A-fragment registers of an m16n8k16 MMA (exact biased integers, see
 // unpack_int4x8_f16 / unpack_int4x8_biased) and multiplies them with the
 // hidden states (B fragments, tokens on the 8-wide side), accumulating in
-// fp32.  The accumulators run in units of the current quantisation group's
-// scale: at the start of each group they are multiplied by the ratio of the
-// previous group's scale to this one's and given the group's bias term, and
-// the last group's scale multiplies the finished residual once.  The rank-r
-// branches follow as extra k steps: int8 codes of A_c (core) or A_w
-// (correction) times the bf16 hi/lo split of t = x V from the pre-pass, the
-// correction in units of the row scale of A_w.  The pre-pass runs as the
-// preceding grid; this kernel starts streaming under programmatic dependent
-// launch and waits for the pre-pass only before the first rank-r stage.
+// fp32.  Each quantisation group starts from its bias term and is promoted
+// by the row's group scale at its end (part sums added into acc); the
+// 64-token instance, with no registers for part sums, keeps its
+// accumulators in units of the current group's scale instead (each group
+// multiplies them by the ratio of the previous scale to its own, and the last
+// scale multiplies the finished residual once).  The rank-r branches follow
+// as extra k steps: int8 codes of A_c (core) or A_w (correction) times the
+// bf16 hi/lo split of t = x V from the pre-pass, the correction promoted by
+// the row scale of A_w.  The pre-pass runs as the preceding grid; this
+// kernel starts streaming under programmatic dependent launch and waits for
+// the pre-pass only before the first rank-r stage.
 //
 // In the paper's packed format (SC4) a group scale is s_row * (q + 1) with a
-// 4-bit code q: the group ratios come from q + 1 (read from the stage's code
-// bytes) and the row scale s_row, which the first rank-r stage carries,
-// multiplies the finished residual once per row.
+// 4-bit code q: the group promotion multiplies by q + 1 (read from the
+// stage's code bytes) and the row scale s_row, which the first rank-r stage
+// carries, multiplies the finished residual once per row.
 #pragma once
 
 #include "device.cuh"
