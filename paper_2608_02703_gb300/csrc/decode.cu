@@ -74,10 +74,24 @@ cudaError_t launch_decode(const DecodeParams &dp, int grid, cudaStream_t s, bool
 // each variant needs the most shared memory.
 cudaError_t prepare_decode(const archead_pack *p) {
   if (!decode_supported(p->d_pad, p->nls_dec, p->g)) return cudaSuccess;
+  // For every instance some M <= 64 selects, the M that needs it most shared
+  // memory (the instance can change with M on heads too wide for x of every
+  // token count to stay resident).
+  constexpr int kVariants = 6;
+  static_assert(kDecStreamedH + 1 == kVariants, "one entry per decode instance");
+  int best_m[kVariants] = {0, 0, 0, 0, 0, 0};
+  size_t best_bytes[kVariants] = {0, 0, 0, 0, 0, 0};
+  for (int M = 1; M <= kDecodeWideTokens; ++M) {
+    const int v = decode_variant(p, M);
+    const int m = std::min(M, variant_tokens(v));
+    const size_t bytes = decode_plan(p->d_pad, p->nls_dec, p->g, m, v).total;
+    if (v >= 0 && v < kVariants && bytes >= best_bytes[v]) best_bytes[v] = bytes, best_m[v] = m;
+  }
   DecodeParams dp = decode_params(p, nullptr, kDecodeWideTokens);
-  for (int M : {8, 16, 32, kDecodeWideTokens}) {
-    dp.variant = decode_variant(p, M);
-    dp.M = std::min(M, variant_tokens(dp.variant));
+  for (int v = 0; v < kVariants; ++v) {
+    if (best_m[v] == 0) continue;
+    dp.variant = v;
+    dp.M = best_m[v];
     const cudaError_t e = launch_decode(dp, 0, nullptr, false);
     if (e != cudaSuccess) return e;
   }

@@ -165,3 +165,34 @@ def test_noalloc_capture_after_warm_up_at_another_token_count():
                         where="capture at M=16 after warm-up at M=1")
     finally:
         pack.close()
+
+
+def test_noalloc_capture_of_the_resident_instance_after_warm_up_at_m8():
+    """d = 8192: eight tokens of x do not stay resident next to a full ring,
+    so M = 8 runs the streamed-x instance and M = 1 the resident one.  A
+    warm-up at M = 8 still prepares the resident instance, and a capture at
+    M = 1 replays against the oracle."""
+    import torch
+
+    shape = HeadShape(V=520, d=8192, core_rank=16, corr_rank=8, group_size=128)
+    head = make_head(shape, seed=19)
+    pack = archead.archead_pack_create(head, shape)
+    try:
+        x8 = gu.to_dev(make_hidden(shape.d, 8, seed=19))
+        y8 = torch.zeros((8, shape.V), dtype=torch.float32, device="cuda")
+        archead.archead_forward_decode_noalloc(pack, x8, 8, y8, archead.OUT_FP32)
+        torch.cuda.synchronize()
+        xd = torch.zeros((1, shape.d), dtype=torch.int16, device="cuda")
+        y = torch.zeros((1, shape.V), dtype=torch.float32, device="cuda")
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            archead.archead_forward_decode_noalloc(pack, xd, 1, y, archead.OUT_FP32)
+        x = make_hidden(shape.d, 1, seed=20)
+        xd.copy_(torch.from_numpy(x.view(np.int16)))
+        g.replay()
+        torch.cuda.synchronize()
+        assert archead.archead_sync_status(pack) == archead.OK
+        gu.check_logits(y.cpu().numpy().astype(np.float64), oracle.logits(head, shape, x),
+                        where="capture at M=1 after warm-up at M=8, d=8192")
+    finally:
+        pack.close()
