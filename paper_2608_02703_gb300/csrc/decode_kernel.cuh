@@ -844,48 +844,48 @@ __global__ void __launch_bounds__(variant_threads(VAR, kSC4), 1) decode_kernel(c
               }
             }
           }
-          continue;
-        }
+        } else {
 #pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-          uint32_t a[4];
-          unpack_int8x8(lw[l][mt].x, lw[l][mt].y, a);
-          if (kb > 0) {  // core columns
-            uint32_t ac[4] = {a[0], a[1], a[2], a[3]};
-            if (kb < 16) {
-              ac[0] &= m0;
-              ac[1] &= m0;
-              ac[2] &= m1;
-              ac[3] &= m1;
-            }
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-              mma_bf16_16816(acc[mt][nt], ac, bh[nt][0], bh[nt][1]);
-              mma_bf16_16816(acc[mt][nt], ac, bl[nt][0], bl[nt][1]);
-            }
-          }
-          if (kb < 16) {  // correction columns
-            if (kb > 0) {
-              a[0] &= ~m0;
-              a[1] &= ~m0;
-              a[2] &= ~m1;
-              a[3] &= ~m1;
-            }
-            if (kRatio && first_corr) {  // continue in units of s_a
-              const float il = __fdividef(1.f, a_lo[mt]), ih = __fdividef(1.f, a_hi[mt]);
+          for (int mt = 0; mt < MT; ++mt) {
+            uint32_t a[4];
+            unpack_int8x8(lw[l][mt].x, lw[l][mt].y, a);
+            if (kb > 0) {  // core columns
+              uint32_t ac[4] = {a[0], a[1], a[2], a[3]};
+              if (kb < 16) {
+                ac[0] &= m0;
+                ac[1] &= m0;
+                ac[2] &= m1;
+                ac[3] &= m1;
+              }
 #pragma unroll
               for (int nt = 0; nt < NT; ++nt) {
-                acc[mt][nt][0] *= il;
-                acc[mt][nt][1] *= il;
-                acc[mt][nt][2] *= ih;
-                acc[mt][nt][3] *= ih;
+                mma_bf16_16816(acc[mt][nt], ac, bh[nt][0], bh[nt][1]);
+                mma_bf16_16816(acc[mt][nt], ac, bl[nt][0], bl[nt][1]);
               }
             }
+            if (kb < 16) {  // correction columns
+              if (kb > 0) {
+                a[0] &= ~m0;
+                a[1] &= ~m0;
+                a[2] &= ~m1;
+                a[3] &= ~m1;
+              }
+              if (kRatio && first_corr) {  // continue in units of s_a
+                const float il = __fdividef(1.f, a_lo[mt]), ih = __fdividef(1.f, a_hi[mt]);
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-              float (&pt)[4] = kRatio ? acc[mt][nt] : part[kRatio ? 0 : mt][kRatio ? 0 : nt];
-              mma_bf16_16816(pt, a, bh[nt][0], bh[nt][1]);
-              mma_bf16_16816(pt, a, bl[nt][0], bl[nt][1]);
+                for (int nt = 0; nt < NT; ++nt) {
+                  acc[mt][nt][0] *= il;
+                  acc[mt][nt][1] *= il;
+                  acc[mt][nt][2] *= ih;
+                  acc[mt][nt][3] *= ih;
+                }
+              }
+#pragma unroll
+              for (int nt = 0; nt < NT; ++nt) {
+                float (&pt)[4] = kRatio ? acc[mt][nt] : part[kRatio ? 0 : mt][kRatio ? 0 : nt];
+                mma_bf16_16816(pt, a, bh[nt][0], bh[nt][1]);
+                mma_bf16_16816(pt, a, bl[nt][0], bl[nt][1]);
+              }
             }
           }
         }
